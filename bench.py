@@ -1,0 +1,420 @@
+"""Benchmark of the STRIDE scoring path on GB300.
+
+One step = one pass of the whole scoring path over the batch-scoring
+workload: 64 trajectories x 8 turns, turn lengths U{64..512} (148,909 rows),
+V = 151,936 bf16 student and teacher logits resident in HBM (90.5 GB, far
+more than L2, so no flush is needed between steps).  A step initialises the
+per-trajectory state and runs stride_score_batch over all rows (per-row
+log-probs, OPD signal, turn statistics, running turn-mean sum, first
+crossing of lambda).
+
+Reported: scored tokens/s (device-timed, CUDA events on the launching
+stream), the same metric end to end through the C ABI from pinned host
+buffers (host->device copy of the step's logits and tokens, device->host
+copy of its results), the roofline of the fused scoring kernel against the
+measured HBM copy bandwidth, and the fp64 CPU oracle timed on this host's
+cores on a bounded sample.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+
+With N > 1 (under torchrun) every rank scores its own replica of the
+workload; there is no collective on the data path ("weak" scaling).
+--impl reference times the oracle (the only reference this path has) on a
+bounded sample per step.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+from pathlib import Path
+
+import numpy as np
+
+ROOT = Path(__file__).resolve().parent
+sys.path.insert(0, str(ROOT))
+
+METRIC = "scored tokens/sec (V=151,936 bf16)"
+UNIT = "tokens/s"
+
+
+def algorithmic_bytes_per_row(V: int, elem: int = 2) -> int:
+    # S row + T row read once, token id read, three fp32 outputs written,
+    # ~8 B amortised per-turn / per-trajectory state and statistics
+    return 2 * V * elem + 4 + 12 + 8
+
+
+def measured_peaks() -> dict:
+    p = ROOT / "MEASURED_PEAKS.json"
+    if p.exists():
+        return json.loads(p.read_text())
+    return {}
+
+
+def kernel_traffic_record() -> tuple[float | None, str]:
+    """DRAM traffic per launch of the fused kernel from the committed ncu
+    summary, valid only while the kernel source is unchanged."""
+    src = ROOT / "paper_2609_14636_gb300" / "csrc"
+    h = hashlib.sha256()
+    for f in ("score_batch.cu", "stride_device.cuh"):
+        h.update((src / f).read_bytes())
+    digest = h.hexdigest()[:16]
+    rec = ROOT / "profiles" / "score_batch_traffic.txt"
+    if not rec.exists():
+        return None, digest
+    kv = {}
+    for line in rec.read_text().splitlines():
+        if ":" in line:
+            k, v = line.split(":", 1)
+            kv[k.strip()] = v.strip()
+    if kv.get("source_sha256_16") != digest:
+        return None, digest
+    try:
+        return float(kv["dram_bytes_per_row"]), digest
+    except (KeyError, ValueError):
+        return None, digest
+
+
+class ClockSampler:
+    """nvidia-smi clock / throttle sampling while the timed region runs."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index = index
+        self.proc = None
+        self.path = Path(os.environ.get("TMPDIR", "/tmp")) / f"stride_clocks_{os.getpid()}.csv"
+
+    def __enter__(self):
+        try:
+            self.f = open(self.path, "w")
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.index}", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-lms", "200"], stdout=self.f, stderr=subprocess.DEVNULL)
+        except (OSError, FileNotFoundError):
+            self.proc = None
+        return self
+
+    def __exit__(self, *a):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+            self.f.close()
+
+    def summary(self) -> dict:
+        if self.proc is None or not self.path.exists():
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["clock sampling unavailable"]}
+        rows = [l.split(",") for l in self.path.read_text().splitlines() if l.strip()]
+        sm, smax, reasons = [], None, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for r in rows:
+            r = [x.strip() for x in r]
+            if len(r) < 9:
+                continue
+            try:
+                sm.append(float(r[1]))
+                smax = float(r[2])
+            except ValueError:
+                continue
+            for n, v in zip(names, r[5:9]):
+                if v.lower().startswith("active"):
+                    reasons.add(n)
+        try:
+            self.path.unlink()
+        except OSError:
+            pass
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": smax,
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+def dist_env():
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return ws, rank, local
+
+
+def cpu_oracle_rate(S_dev, T_dev, tok_dev, lay, lam, budget_s: float, chunk: int = 1024) -> dict:
+    """Oracle rows/s on a bounded sample: consecutive 1,024-row chunks of the
+    workload, copied device->host, until ~budget_s of oracle time."""
+    import oracle
+    import torch
+
+    lib = oracle.get()
+    threads = oracle.default_threads()
+    rows_done, t_oracle = 0, 0.0
+    R = S_dev.shape[0]
+    r0 = 0
+    while t_oracle < budget_s and r0 < R:
+        r1 = min(R, r0 + chunk)
+        Sh = S_dev[r0:r1].view(torch.int16).cpu().numpy().view(np.uint16)
+        Th = T_dev[r0:r1].view(torch.int16).cpu().numpy().view(np.uint16)
+        th = tok_dev[r0:r1].cpu().numpy()
+        t0 = time.perf_counter()
+        o = lib.row_logprobs(Sh, Th, th, nthreads=threads)
+        t_oracle += time.perf_counter() - t0
+        rows_done += r1 - r0
+        r0 = r1
+        del Sh, Th, o
+    return {"value": rows_done / t_oracle, "unit": UNIT, "cores": threads, "kind": "oracle",
+            "sample": f"first {rows_done} rows of the workload (fp64 log-softmax gather of S and T, "
+                      f"{threads} threads), {t_oracle:.1f} s"}
+
+
+def run_reference(args) -> None:
+    """--impl reference: the fp64 CPU oracle, as it stands, on a bounded
+    sample of the workload per step (1,024 rows of its logits)."""
+    ws, rank, local = dist_env()
+    if rank != 0:
+        return
+    import torch
+
+    import oracle
+    import synth
+
+    w = synth.batch_scoring()
+    rows = 1024
+    dev = "cuda" if torch.cuda.is_available() else "cpu"
+    S, T, tok = synth.generate_rows(w.recipe, 0, rows, device=dev)
+    Sh = S.view(torch.int16).cpu().numpy().view(np.uint16)
+    Th = T.view(torch.int16).cpu().numpy().view(np.uint16)
+    th = tok.cpu().numpy()
+    lay = synth.layout_from_turn_lengths([[rows]])
+    lib = oracle.get()
+    threads = oracle.default_threads()
+    lam = float(load_lambda(w)[0])
+
+    def step():
+        o = lib.row_logprobs(Sh, Th, th, nthreads=threads)
+        lib.scan_batch(o["logp_t"], o["d"], lay.traj_row_off, lay.turn_row_off, lay.traj_turn_off, 0, lam)
+
+    for _ in range(args.warmup):
+        step()
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        step()
+    dt = time.perf_counter() - t0
+    value = rows * args.steps / dt
+    line = {"metric": METRIC, "value": value, "unit": UNIT, "impl": "reference", "n_gpus": ws,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * dt / args.steps,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic", "config": {"workload": w.name, "sample_rows_per_step": rows},
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": threads, "kind": "oracle",
+                             "sample": f"{rows} rows of the workload per step, fp64 oracle, {threads} threads"},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+def load_lambda(w) -> np.ndarray:
+    """Per-trajectory lambda: the oracle calibration of the workload
+    (tests/golden/lambda_calibration.json), else its provisional value."""
+    import synth
+
+    return np.full(w.layout.n_traj, np.float32(synth.workload_lambda(w.name)), np.float32)
+
+
+def main() -> None:
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--cpu-budget", type=float, default=12.0, help="seconds of oracle time for cpu_baseline")
+    ap.add_argument("--e2e-rows", type=int, default=8192)
+    ap.add_argument("--max-rows", type=int, default=0,
+                    help="score only the leading whole trajectories that fit (small profiling cases)")
+    args = ap.parse_args()
+    if args.impl == "reference":
+        run_reference(args)
+        return
+
+    import torch
+
+    ws, rank, local = dist_env()
+    if ws > 1:
+        import torch.distributed as dist
+
+        dist.init_process_group("nccl")
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+
+    import paper_2609_14636_gb300 as stride
+    import synth
+
+    w = synth.batch_scoring()
+    lay = w.layout
+    if args.max_rows > 0:
+        lay = synth.sub_layout(lay, synth.first_trajectories(lay, args.max_rows))
+    R, V = lay.rows, w.recipe.V
+    lam = load_lambda(w)[: lay.n_traj]
+
+    # ---- workload resident in HBM --------------------------------------
+    S = torch.empty((R, V), dtype=torch.bfloat16, device=dev)
+    T = torch.empty((R, V), dtype=torch.bfloat16, device=dev)
+    tok = torch.empty(R, dtype=torch.int32, device=dev)
+    t_gen = time.perf_counter()
+    CH = 8192
+    for r0 in range(0, R, CH):
+        r1 = min(R, r0 + CH)
+        synth.generate_rows(w.recipe, r0, r1 - r0, device=dev, out_S=S[r0:r1], out_T=T[r0:r1], out_tok=tok[r0:r1])
+    torch.cuda.synchronize()
+    t_gen = time.perf_counter() - t_gen
+    offs = [torch.from_numpy(a).to(dev) for a in (lay.traj_row_off, lay.turn_row_off, lay.traj_turn_off)]
+    lam_d = torch.from_numpy(lam).to(dev)
+    st = stride.new_state(lay.n_traj, dev)
+    ts = stride.new_turn_stats(lay.n_turns, dev)
+    out = {k: torch.empty(R, dtype=torch.float32, device=dev) for k in ("logp_s", "logp_t", "opd")}
+    status = torch.zeros(1, dtype=torch.int32, device=dev)
+    wsb = torch.empty(stride.stride_score_batch_workspace_size(R), dtype=torch.uint8, device=dev)
+    stream = torch.cuda.current_stream()
+
+    def step(ev=None):
+        stride.stride_state_init(st, lay.n_traj, stream)
+        if ev is not None:
+            ev[0].record(stream)
+        stride.stride_score_batch(S, T, tok, *offs, 0, R, stride.TURN_MEAN, lam_d, st, out=out, turn_stats=ts,
+                                  dev_status=status, workspace=wsb, stream=stream)
+        if ev is not None:
+            ev[1].record(stream)
+
+    for _ in range(max(3, args.warmup)):
+        step()
+    torch.cuda.synchronize()
+    if int(status.item()) != 0:
+        raise RuntimeError(f"device status {int(status.item())} after warm-up")
+    early = stride.state_to_numpy(st)[: lay.n_traj]
+    n_turns_traj = np.diff(lay.traj_turn_off)
+    early_frac = float(np.mean((early["stop_turn"] >= 0) & (early["stop_turn"] < n_turns_traj - 1)))
+
+    # ---- device-timed steps ---------------------------------------------
+    kev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    if ws > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    with ClockSampler(local) as clk:
+        time.sleep(0.25)
+        e0.record(stream)
+        for i in range(args.steps):
+            step(kev[i])
+        e1.record(stream)
+        torch.cuda.synchronize()
+        time.sleep(0.05)
+    if ws > 1:
+        dist.barrier()
+    ms_total = e0.elapsed_time(e1)
+    k_ms = [a.elapsed_time(b) for a, b in kev]
+    if ws > 1:
+        t = torch.tensor([ms_total], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms_total = float(t.item())
+    ms_step = ms_total / args.steps
+    value = ws * R / (ms_step * 1e-3)
+
+    # ---- roofline of the fused kernel -------------------------------------
+    peaks = measured_peaks()
+    peak = peaks.get("hbm_gbs", 6800.0)
+    bpr = algorithmic_bytes_per_row(V)
+    k_avg = statistics.mean(k_ms)
+    achieved = bpr * R / (k_avg * 1e-3) / 1e9
+    dram_per_row, digest = kernel_traffic_record()
+    roofline = {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s", "frac": achieved / peak,
+                "traffic": None if dram_per_row is None else dram_per_row * R,
+                "algorithmic_bytes_per_launch": bpr * R, "kernel_ms_mean": k_avg,
+                "kernel_ms_min": min(k_ms), "kernel": "score_batch_kernel<bf16,vec>",
+                "peak_source": "MEASURED_PEAKS.json hbm_gbs (of measured)" if "hbm_gbs" in peaks else "fallback 6.8 TB/s"}
+
+    # ---- end to end from pinned host buffers ------------------------------
+    e2e = None
+    if rank == 0 or ws > 1:
+        # the first trajectories up to e2e_rows rows, as a caller holding them in host memory would
+        n_tr = int(np.searchsorted(lay.traj_row_off, args.e2e_rows, side="right") - 1)
+        n_tr = max(1, min(n_tr, lay.n_traj))
+        Re = int(lay.traj_row_off[n_tr])
+        n_tu = int(lay.traj_turn_off[n_tr])
+        hS = torch.empty((Re, V), dtype=torch.bfloat16, pin_memory=True)
+        hT = torch.empty((Re, V), dtype=torch.bfloat16, pin_memory=True)
+        hk = torch.empty(Re, dtype=torch.int32, pin_memory=True)
+        hS.copy_(S[:Re])
+        hT.copy_(T[:Re])
+        hk.copy_(tok[:Re])
+        hout = {k: torch.empty(Re, dtype=torch.float32, pin_memory=True) for k in out}
+        hst = torch.empty((n_tr, 56), dtype=torch.uint8, pin_memory=True)
+        hts = torch.empty((n_tu, 32), dtype=torch.uint8, pin_memory=True)
+        dS, dT, dk = S[:Re], T[:Re], tok[:Re]  # device landing buffers (the resident workload's first rows)
+        eoffs = [torch.from_numpy(a).to(dev) for a in (lay.traj_row_off[: n_tr + 1], lay.turn_row_off[: n_tu + 1],
+                                                        lay.traj_turn_off[: n_tr + 1])]
+        est = stride.new_state(n_tr, dev)
+        ets = stride.new_turn_stats(n_tu, dev)
+        eout = {k: v[:Re] for k, v in out.items()}
+
+        def e2e_step():
+            dS.copy_(hS, non_blocking=True)
+            dT.copy_(hT, non_blocking=True)
+            dk.copy_(hk, non_blocking=True)
+            stride.stride_state_init(est, n_tr, stream)
+            stride.stride_score_batch(dS, dT, dk, *eoffs, 0, Re, stride.TURN_MEAN, lam_d[:n_tr], est, out=eout,
+                                      turn_stats=ets, dev_status=status, workspace=wsb, stream=stream)
+            for k in hout:
+                hout[k].copy_(eout[k], non_blocking=True)
+            hst.copy_(est[:n_tr], non_blocking=True)
+            hts.copy_(ets[:n_tu], non_blocking=True)
+
+        for _ in range(2):
+            e2e_step()
+        torch.cuda.synchronize()
+        n_e = max(2, min(args.steps, 5))
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        for _ in range(n_e):
+            e2e_step()
+        b.record(stream)
+        torch.cuda.synchronize()
+        e_ms = a.elapsed_time(b) / n_e
+        h2d = 2 * Re * V * 2 + Re * 4
+        d2h = Re * 4 * len(hout) + n_tr * 56 + n_tu * 32
+        e2e = {"value": ws * Re / (e_ms * 1e-3), "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
+               "ms_per_step": e_ms, "sample": f"first {n_tr} trajectories ({Re} rows) of the workload held in pinned "
+                                              f"host memory; H2D of S, T, tokens and D2H of per-row outputs, state "
+                                              f"and turn stats inside the timed region"}
+        del hS, hT
+
+    # ---- oracle on this host's cores (rank 0, N = 1 only) ------------------
+    cpu = None
+    if rank == 0 and ws == 1:
+        cpu = cpu_oracle_rate(S, T, tok, lay, lam, args.cpu_budget)
+
+    if rank == 0:
+        clocks = clk.summary()
+        line = {
+            "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws, "steps": args.steps,
+            "warmup": max(3, args.warmup), "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+            "config": {"workload": w.name if args.max_rows <= 0 else f"{w.name} (first {lay.n_traj} trajectories)",
+                       "trajectories": lay.n_traj, "turns": lay.n_turns, "rows": R,
+                       "vocab": V, "logits": "bf16 student + bf16 teacher, resident in HBM",
+                       "bytes_resident": 2 * R * V * 2, "stop_mode": "turn_mean",
+                       "lambda": float(lam[0]), "early_stop_fraction": early_frac,
+                       "l2": f"inputs ({2 * R * V * 2 / 1e9:.1f} GB) larger than L2 (129 MB): no flush",
+                       "parallelism": f"replicas x{ws}" if ws > 1 else "single GPU",
+                       "generation_s": t_gen},
+            "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e, "clocks": clocks,
+            "gpu_launches": 2 * args.steps,
+        }
+        print(json.dumps(line), flush=True)
+    if ws > 1:
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,227 @@
+/*
+ * stride.h -- C ABI of the STRIDE scoring path (arXiv 2609.14636) on one
+ * NVIDIA GB300 (sm_103a).
+ *
+ * The library computes the per-token teacher/student scoring that STRIDE's
+ * adaptive early stopping and prefix buffer act on:
+ *
+ *   log pi_S(y_t), log pi_T(y_t)   log-softmax over the vocabulary, gathered
+ *                                  at the sampled token (Eq. 1, Eq. 4);
+ *   d_t = log pi_S - log pi_T      the per-token OPD signal, = -r_t of Eq. 1
+ *                                  (the per-token KL estimate of Sec. 3.2);
+ *   l_k                            per-turn mean teacher log-prob (Eq. 4);
+ *   first crossing                 the first turn K* whose running sum of
+ *                                  turn means, over the newly generated turns
+ *                                  only, falls below lambda (Eq. 5 with the
+ *                                  prefix-buffer offset of Sec. 4.1), or the
+ *                                  first token whose running teacher log-prob
+ *                                  falls below lambda (Sec. 5.5);
+ *   k*, K_max                      the weakest correct turn of Eq. 6 behind
+ *                                  the quality gate of Sec. 4.2.
+ *
+ * Conventions shared by every entry point
+ * ---------------------------------------
+ * - All array pointers are DEVICE pointers owned by the caller (allocate them
+ *   with cudaMalloc, torch, ...).  Struct pointers passed as "host struct" are
+ *   read on the host during the call only.  The library allocates no memory;
+ *   scratch space is a caller-provided workspace whose size a *_workspace_size
+ *   query returns.
+ * - Every compute call is asynchronous on the caller's `stream` (a
+ *   cudaStream_t passed as void*; NULL = the legacy default stream) and
+ *   returns a stride_status after host-side argument checks and the launch.
+ *   A non-zero return means nothing was launched (or the launch failed:
+ *   STRIDE_ERR_CUDA).
+ * - Errors found on the device are OR-ed into the caller's int32 `dev_status`
+ *   word (STRIDE_DEV_* bits; nullable), readable after the stream has
+ *   synchronised.  Kernels never trap: a bad row gets NaN outputs.
+ * - Logit rows are row-major with a row stride `ld` (elements, ld >= V).
+ *   Rows whose address and stride are 16-byte aligned take the vectorised
+ *   path; others take a scalar path with the same results.
+ * - Turn and row indices reported per trajectory are 0-based and local to the
+ *   trajectory.  The paper's turns are 1-based, so the returned k* equals its
+ *   K0 = k* - 1 (Algorithm 1): the number of turns reused as context.
+ * - Every compute call is a plain kernel launch (plus cudaMemsetAsync of the
+ *   workspace for stride_score_batch), so a sequence of calls can be captured
+ *   in a CUDA graph.
+ * - The library is built for sm_103a only; on another device the calls return
+ *   STRIDE_ERR_UNSUPPORTED_DEVICE.  There is no CPU fallback.
+ */
+#ifndef STRIDE_H_
+#define STRIDE_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define STRIDE_ABI_VERSION 1
+
+#if defined(__GNUC__)
+#define STRIDE_API __attribute__((visibility("default")))
+#else
+#define STRIDE_API
+#endif
+
+/* ---- return codes ------------------------------------------------------ */
+typedef enum stride_status {
+  STRIDE_OK = 0,
+  STRIDE_ERR_INVALID_ARG = 1,        /* a pointer, size, mode or layout is invalid */
+  STRIDE_ERR_UNSUPPORTED_DTYPE = 2,  /* dtype is not BF16 or F32 */
+  STRIDE_ERR_WORKSPACE = 3,          /* workspace missing, too small or misaligned */
+  STRIDE_ERR_CUDA = 4,               /* a CUDA runtime call or launch failed */
+  STRIDE_ERR_UNSUPPORTED_DEVICE = 5  /* current device is not compute capability 10.3 */
+} stride_status;
+
+/* ---- device status bits (OR-ed into *dev_status) ----------------------- */
+#define STRIDE_DEV_TOKEN_RANGE 0x1 /* a token is outside [0, V): that row is NaN */
+#define STRIDE_DEV_BAD_LAYOUT 0x2  /* offsets not monotone, an empty turn, or a row outside its turn */
+#define STRIDE_DEV_TIMEOUT 0x4     /* a bounded device-side wait gave up (results of that call are invalid) */
+
+/* ---- enums ---------------------------------------------------------------- */
+#define STRIDE_DTYPE_BF16 0 /* logits are bfloat16 */
+#define STRIDE_DTYPE_F32 1  /* logits are float32 */
+
+#define STRIDE_STOP_TURN_MEAN 0 /* Eq. 5: running sum of per-turn means l_k, tested at turn ends */
+#define STRIDE_STOP_TOKEN_SUM 1 /* Sec. 5.5: running sum of token log-probs, tested at every token */
+
+/* ---- per-trajectory / per-rollout carried state (56 bytes) ---------------
+ * Initialise with stride_state_init.  It is both the carry between calls
+ * (chunked batch scoring, decode steps) and the per-trajectory result.
+ * A trajectory's running sum starts from `cum` at its first row (0 after
+ * init), which is how the prefix-buffer offset is expressed: pass only the
+ * newly generated turns of a restarted rollout (Sec. 4.1; Algorithm 1). */
+typedef struct stride_scan_state {
+  double cum;          /* running sum through the last scored token (Eq. 5 LHS or token sum) */
+  double turn_sum_t;   /* open turn: sum of log pi_T so far */
+  double turn_sum_d;   /* open turn: sum of d so far */
+  int64_t rows_seen;   /* tokens of this trajectory scored so far */
+  int64_t stop_row;    /* token position (trajectory-local) of the first crossing; -1 = none */
+  int32_t stop_turn;   /* turn (trajectory-local, 0-based) of the first crossing; -1 = none */
+  int32_t turn_tokens; /* tokens in the open turn */
+  int32_t turn_idx;    /* index of the open turn (trajectory-local) */
+  int32_t stopped;     /* non-zero once the stop rule has fired */
+} stride_scan_state;
+
+/* ---- per-turn statistics (32 bytes) --------------------------------------- */
+typedef struct stride_turn_stats {
+  double sum_t;  /* sum of log pi_T over the turn's tokens */
+  double sum_d;  /* sum of d over the turn's tokens (turn mean KL = sum_d / n, Sec. 3.2) */
+  double cum;    /* running sum after this turn (Eq. 5 LHS; token sum at the turn's end in TOKEN_SUM) */
+  float mean_t;  /* l_k = sum_t / n (Eq. 4), rounded to fp32 */
+  int32_t n;     /* tokens in the turn (n_k) */
+} stride_turn_stats;
+
+/* ---- optional per-row outputs (host struct of device pointers) ------------
+ * Each pointer is nullable; a non-NULL pointer receives one float per row. */
+typedef struct stride_row_outputs {
+  float* logp_s; /* log pi_S(y_t) */
+  float* logp_t; /* log pi_T(y_t) */
+  float* opd;    /* d_t = log pi_S(y_t) - log pi_T(y_t) = -r_t (Eq. 1) */
+  float* lse_s;  /* log sum_j exp(S_j) */
+  float* lse_t;  /* log sum_j exp(T_j) */
+  float* x_s;    /* S[y_t], the gathered student logit (exact) */
+  float* x_t;    /* T[y_t], the gathered teacher logit (exact) */
+} stride_row_outputs;
+
+/* Initialise n states: zeros, stop_row = -1, stop_turn = -1.
+ * state: device [n].  Asynchronous on stream. */
+STRIDE_API int stride_state_init(stride_scan_state* state, int32_t n, void* stream);
+
+/* Workspace bytes stride_score_batch needs for a window of `window_rows`
+ * rows (0 for an empty window).  The workspace must be 256-byte aligned. */
+STRIDE_API size_t stride_score_batch_workspace_size(int64_t window_rows);
+
+/* Score a window of rows of ragged trajectories, with turn offsets.
+ * (Eq. 1, Eq. 4, Eq. 5 with the prefix-buffer offset, Sec. 5.5.)
+ *
+ * Global layout (device arrays, int64 rows): trajectory i owns rows
+ * [traj_row_off[i], traj_row_off[i+1]) and turns [traj_turn_off[i],
+ * traj_turn_off[i+1]); turn k owns rows [turn_row_off[k], turn_row_off[k+1]).
+ * Every turn must hold at least one row (Eq. 4 divides by n_k).
+ * traj_row_off[0] <= row_begin <= row_end <= traj_row_off[n_traj].
+ *
+ * This call scores global rows [row_begin, row_end): S, T point at the logits
+ * of row_begin ([row_end-row_begin, ld], dtype STRIDE_DTYPE_*), tokens at its
+ * token (int32 [row_end-row_begin]).  Calling with consecutive windows on one
+ * stream, with the same `state`, gives the same results as one call over all
+ * rows: the state carries each trajectory's running sum and open-turn sums
+ * across window edges.
+ *
+ * stop_mode: STRIDE_STOP_TURN_MEAN or STRIDE_STOP_TOKEN_SUM.  lambda: device
+ * float [n_traj] per-trajectory thresholds, or NULL to use lambda_all for
+ * every trajectory (the scale of lambda depends on the generation unit and is
+ * chosen per domain, Sec. 4.1).  The test is strict: sum < lambda.  The
+ * token or turn that triggers is retained (Sec. 4.1).  Later turns are still
+ * scored; the stop fields keep the first crossing.
+ *
+ * state: device [n_traj], in/out (see stride_scan_state).
+ * out: host struct of optional per-row outputs indexed by (row - row_begin); NULL for none.
+ * turn_stats: device [n_turns] or NULL; turn k is written by the call that
+ * scores its last row.
+ * dev_status: device int32 or NULL.
+ * workspace: device, >= stride_score_batch_workspace_size(row_end-row_begin)
+ * bytes, 256-byte aligned; it is cleared by the call, holds nothing between
+ * calls, and one workspace must not be shared by calls that overlap in time.
+ * Returns STRIDE_OK or an error code; launches nothing when row_begin == row_end. */
+STRIDE_API int stride_score_batch(const void* S, const void* T, int32_t dtype, int64_t ld, int64_t V,
+                       const int32_t* tokens, const int64_t* traj_row_off,
+                       const int64_t* turn_row_off, const int32_t* traj_turn_off, int32_t n_traj,
+                       int32_t n_turns, int64_t row_begin, int64_t row_end, int32_t stop_mode,
+                       const float* lambda, float lambda_all, stride_scan_state* state,
+                       const stride_row_outputs* out, stride_turn_stats* turn_stats,
+                       int32_t* dev_status, void* workspace, size_t workspace_bytes,
+                       void* stream);
+
+/* One decode step over B rollouts (Algorithm 1, inner turn loop, one
+ * generated token per rollout).
+ *
+ * S, T: [B, ld] logits of this step's token of each rollout; tokens: int32
+ * [B]; turn_end: uint8 [B], non-zero when this token closes the rollout's
+ * current turn.  state: device [B], in/out.  A rollout whose state.stopped is
+ * set is masked: its logits are not read, its state is not changed, its
+ * per-row outputs are NaN.  For an active rollout the token is scored, the
+ * open turn accumulates, and:
+ *   TOKEN_SUM: cum += log pi_T; stop if cum < lambda;
+ *   TURN_MEAN: at a turn end, l = turn_sum_t / turn_tokens (Eq. 4),
+ *              cum += l, stop if cum < lambda (Eq. 5).
+ * stopped_now: uint8 [B] or NULL, 1 where the rule fired at this step.
+ * turn_out: device [B] or NULL: the stats of the turn closed at this step
+ * (n = 0 where none closed).  lambda / lambda_all as for stride_score_batch.
+ * The call needs no workspace. */
+STRIDE_API int stride_score_step(const void* S, const void* T, int32_t dtype, int64_t ld, int64_t V,
+                      const int32_t* tokens, const uint8_t* turn_end, int32_t B,
+                      int32_t stop_mode, const float* lambda, float lambda_all,
+                      stride_scan_state* state, const stride_row_outputs* out,
+                      uint8_t* stopped_now, stride_turn_stats* turn_out, int32_t* dev_status,
+                      void* stream);
+
+/* Restart choice over N stored trajectory records (Sec. 4.2 steps 1-2,
+ * Eq. 6, Algorithm 1).
+ *
+ * turn_mean: float [N, T_max] row-major (entry i's per-turn l_k); n_turns:
+ * int32 [N] (0 <= n_turns[i] <= T_max); correct: uint8 [N, T_max] or NULL
+ * (an external correctness mask ANDed with the gate).
+ *   correct_k = (correct == NULL || correct[i,k]) && (turn_mean[i,k] > alpha)
+ *   K_max     = length of the longest all-correct run starting at turn 0
+ *   k*        = argmin_{0 <= k < K_max} turn_mean[i,k], lowest index on ties
+ *   K_max = 0 gives k* = 0 (no reusable prefix).
+ * alpha = -INFINITY disables the gate (the paper's math setting; App. A uses
+ * alpha = -0.8 for agentic runs).  NaN means are never correct.
+ * k_star, k_max: int32 [N] outputs.  k_star is 0-based and equals K0. */
+STRIDE_API int stride_select_restart(const float* turn_mean, const int32_t* n_turns, const uint8_t* correct,
+                          float alpha, int32_t N, int32_t T_max, int32_t* k_star,
+                          int32_t* k_max, void* stream);
+
+/* Human-readable name of a stride_status code (static string). */
+STRIDE_API const char* stride_status_string(int code);
+
+/* STRIDE_ABI_VERSION of the loaded library. */
+STRIDE_API int stride_abi_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* STRIDE_H_ */

@@ -73,20 +73,21 @@ class OracleLib:
         """Per-row fp64 log-probs of ``tokens`` under logits S (student), T (teacher).
 
         S, T: 2-D arrays [rows, ld]; ``np.uint16`` holds raw bf16 bits,
-        ``np.float32`` is fp32.  V defaults to ld.  Returns a dict of fp64
+        ``np.float32`` is fp32.  S may be None (teacher only; the student
+        outputs are NaN).  V defaults to ld.  Returns a dict of fp64
         arrays logp_s, logp_t, d, lse_s, lse_t, x_s, x_t and the return code.
         """
-        if S.dtype == np.uint16:
+        if T.dtype == np.uint16:
             dt = DTYPE_BF16
-        elif S.dtype == np.float32:
+        elif T.dtype == np.float32:
             dt = DTYPE_F32
         else:
-            raise TypeError(f"unsupported logit dtype {S.dtype}")
-        if T.dtype != S.dtype or S.shape != T.shape or S.ndim != 2:
-            raise ValueError("S and T must be 2-D arrays of one dtype and shape")
-        S = np.ascontiguousarray(S)
+            raise TypeError(f"unsupported logit dtype {T.dtype}")
+        if T.ndim != 2 or (S is not None and (S.dtype != T.dtype or S.shape != T.shape)):
+            raise ValueError("S and T must be 2-D arrays of one dtype and shape (S may be None)")
+        S = None if S is None else np.ascontiguousarray(S)
         T = np.ascontiguousarray(T)
-        rows, ld = S.shape
+        rows, ld = T.shape
         V = ld if V is None else int(V)
         tok = np.ascontiguousarray(tokens, dtype=np.int32)
         if tok.shape != (rows,):

@@ -106,11 +106,11 @@ static void* rows_worker(void* arg) {
   rows_job* jb = (rows_job*)arg;
   for (int64_t r = jb->r0; r < jb->r1; ++r) {
     int32_t y = jb->tokens[r];
-    double ls = row_lse(jb->S, jb->dtype, jb->ld, jb->V, r);
+    double ls = jb->S ? row_lse(jb->S, jb->dtype, jb->ld, jb->V, r) : NAN;
     double lt = row_lse(jb->T, jb->dtype, jb->ld, jb->V, r);
     double xs = NAN, xt = NAN, ps = NAN, pt = NAN;
     if (y >= 0 && (int64_t)y < jb->V) {
-      xs = logit_at(jb->S, jb->dtype, jb->ld, r, y);
+      xs = jb->S ? logit_at(jb->S, jb->dtype, jb->ld, r, y) : NAN;
       xt = logit_at(jb->T, jb->dtype, jb->ld, r, y);
       ps = xs - ls; /* log pi_S(y_t) */
       pt = xt - lt; /* log pi_T(y_t) */
@@ -130,6 +130,7 @@ static void* rows_worker(void* arg) {
 
 /* Per-row log-probabilities of the sampled token under student S and teacher T.
  * S, T: [rows, ld] row-major, dtype bf16 (raw uint16 bits) or fp32.
+ * S may be NULL (teacher only: student outputs are NaN).
  * Any output pointer may be NULL.  Rows are split across nthreads threads;
  * each row is computed independently, so the thread count does not change
  * any result. */
@@ -137,7 +138,7 @@ int oracle_row_logprobs(const void* S, const void* T, int dtype, int64_t ld, int
                         const int32_t* tokens, int64_t rows, double* logp_s, double* logp_t,
                         double* d, double* lse_s, double* lse_t, double* x_s, double* x_t,
                         int nthreads) {
-  if (!S || !T || !tokens || V < 1 || ld < V || rows < 0) return ORACLE_ERR_ARG;
+  if (!T || !tokens || V < 1 || ld < V || rows < 0) return ORACLE_ERR_ARG;
   if (dtype != ORACLE_DTYPE_BF16 && dtype != ORACLE_DTYPE_F32) return ORACLE_ERR_ARG;
   if (nthreads < 1) nthreads = 1;
   if (nthreads > 1024) nthreads = 1024;

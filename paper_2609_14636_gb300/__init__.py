@@ -1,0 +1,269 @@
+"""STRIDE scoring path on one GB300 (arXiv 2609.14636): Python binding.
+
+A thin ctypes layer over ``libstride.so`` (include/stride.h).  The functions
+keep the C names and argument order; they take torch CUDA tensors, check
+their dtype/device/shape, pass raw device pointers and the current CUDA
+stream, and raise :class:`StrideError` on a non-zero status.  Every step of
+the scoring path runs in the library's CUDA kernels: there is no Python or
+CPU fallback, and importing this package fails if the library is missing
+and cannot be built.
+
+Per-trajectory state and per-turn statistics are opaque byte tensors
+(``[n, 56]`` and ``[n, 32]`` uint8) laid out as ``stride_scan_state`` and
+``stride_turn_stats``; :func:`state_to_numpy` / :func:`turn_stats_to_numpy`
+view copies of them as numpy structured arrays.
+"""
+from __future__ import annotations
+
+import ctypes
+from pathlib import Path
+
+import numpy as np
+
+from . import _build
+
+__all__ = [
+    "StrideError", "STATE_DTYPE", "TURN_STATS_DTYPE", "DTYPE_BF16", "DTYPE_F32", "TURN_MEAN",
+    "TOKEN_SUM", "DEV_TOKEN_RANGE", "DEV_BAD_LAYOUT", "DEV_TIMEOUT", "lib", "new_state",
+    "new_turn_stats", "state_to_numpy", "turn_stats_to_numpy", "stride_state_init",
+    "stride_score_batch_workspace_size", "stride_score_batch", "stride_score_step",
+    "stride_select_restart", "stride_status_string", "stride_abi_version", "ROW_OUTPUT_KEYS",
+]
+
+DTYPE_BF16, DTYPE_F32 = 0, 1
+TURN_MEAN, TOKEN_SUM = 0, 1
+DEV_TOKEN_RANGE, DEV_BAD_LAYOUT, DEV_TIMEOUT = 0x1, 0x2, 0x4
+ROW_OUTPUT_KEYS = ("logp_s", "logp_t", "opd", "lse_s", "lse_t", "x_s", "x_t")
+
+STATE_DTYPE = np.dtype([("cum", "<f8"), ("turn_sum_t", "<f8"), ("turn_sum_d", "<f8"),
+                        ("rows_seen", "<i8"), ("stop_row", "<i8"), ("stop_turn", "<i4"),
+                        ("turn_tokens", "<i4"), ("turn_idx", "<i4"), ("stopped", "<i4")])
+TURN_STATS_DTYPE = np.dtype([("sum_t", "<f8"), ("sum_d", "<f8"), ("cum", "<f8"),
+                             ("mean_t", "<f4"), ("n", "<i4")])
+assert STATE_DTYPE.itemsize == 56 and TURN_STATS_DTYPE.itemsize == 32
+
+
+class StrideError(RuntimeError):
+    def __init__(self, fn: str, code: int):
+        super().__init__(f"{fn}: {stride_status_string(code)} (code {code})")
+        self.code = code
+
+
+class _RowOutputs(ctypes.Structure):
+    _fields_ = [(k, ctypes.c_void_p) for k in ROW_OUTPUT_KEYS]
+
+
+_LIB = None
+
+
+def lib() -> ctypes.CDLL:
+    """The loaded libstride.so (built in-tree on first use if absent)."""
+    global _LIB
+    if _LIB is None:
+        path = _build.LIB
+        if not _build.up_to_date():
+            _build.build()
+        if not Path(path).exists():
+            raise ImportError(f"libstride.so not found at {path}")
+        L = ctypes.CDLL(str(path))
+        P, i32, i64, f32, sz = ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64, ctypes.c_float, ctypes.c_size_t
+        L.stride_state_init.argtypes = [P, i32, P]
+        L.stride_score_batch_workspace_size.argtypes = [i64]
+        L.stride_score_batch_workspace_size.restype = sz
+        L.stride_score_batch.argtypes = [P, P, i32, i64, i64, P, P, P, P, i32, i32, i64, i64, i32, P, f32,
+                                         P, P, P, P, P, sz, P]
+        L.stride_score_step.argtypes = [P, P, i32, i64, i64, P, P, i32, i32, P, f32, P, P, P, P, P, P]
+        L.stride_select_restart.argtypes = [P, P, P, f32, i32, i32, P, P, P]
+        L.stride_status_string.argtypes = [ctypes.c_int]
+        L.stride_status_string.restype = ctypes.c_char_p
+        L.stride_abi_version.restype = ctypes.c_int
+        for fn in ("stride_state_init", "stride_score_batch", "stride_score_step", "stride_select_restart"):
+            getattr(L, fn).restype = ctypes.c_int
+        _LIB = L
+    return _LIB
+
+
+def stride_status_string(code: int) -> str:
+    return lib().stride_status_string(int(code)).decode()
+
+
+def stride_abi_version() -> int:
+    return int(lib().stride_abi_version())
+
+
+# ---------------------------------------------------------------------------
+# marshalling helpers
+# ---------------------------------------------------------------------------
+def _torch():
+    import torch
+
+    return torch
+
+
+def _stream(stream) -> int:
+    torch = _torch()
+    if stream is None:
+        return torch.cuda.current_stream().cuda_stream
+    if isinstance(stream, int):
+        return stream
+    return stream.cuda_stream
+
+
+def _dev(t, name: str, dtype=None, numel: int | None = None, optional: bool = False):
+    if t is None:
+        if optional:
+            return None
+        raise ValueError(f"{name} is required")
+    torch = _torch()
+    if not isinstance(t, torch.Tensor) or not t.is_cuda:
+        raise TypeError(f"{name} must be a CUDA tensor")
+    if dtype is not None and t.dtype != dtype:
+        raise TypeError(f"{name} must be {dtype}, got {t.dtype}")
+    if not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+    if numel is not None and t.numel() < numel:
+        raise ValueError(f"{name} holds {t.numel()} elements, needs {numel}")
+    return t.data_ptr()
+
+
+def _logits(S, T):
+    torch = _torch()
+    for name, x in (("S", S), ("T", T)):
+        if not isinstance(x, torch.Tensor) or not x.is_cuda or x.dim() != 2 or x.stride(1) != 1:
+            raise TypeError(f"{name} must be a 2-D CUDA tensor with unit column stride")
+    if S.dtype != T.dtype or S.shape != T.shape or S.stride(0) != T.stride(0):
+        raise ValueError("S and T must share dtype, shape and row stride")
+    if S.dtype == torch.bfloat16:
+        dt = DTYPE_BF16
+    elif S.dtype == torch.float32:
+        dt = DTYPE_F32
+    else:
+        raise TypeError(f"logits must be bfloat16 or float32, got {S.dtype}")
+    return dt, S.stride(0)
+
+
+def _row_outputs(out: dict | None, rows: int):
+    if not out:
+        return None
+    torch = _torch()
+    ro = _RowOutputs()
+    for k, v in out.items():
+        if k not in ROW_OUTPUT_KEYS:
+            raise KeyError(f"unknown row output {k!r}")
+        setattr(ro, k, _dev(v, k, torch.float32, rows))
+    return ctypes.byref(ro)
+
+
+def _lambda(lam, n: int):
+    torch = _torch()
+    if isinstance(lam, torch.Tensor):
+        return _dev(lam, "lambda", torch.float32, n), float("nan")
+    return None, float(lam)
+
+
+def _check(fn: str, rc: int):
+    if rc != 0:
+        raise StrideError(fn, rc)
+
+
+# ---------------------------------------------------------------------------
+# state / stats buffers
+# ---------------------------------------------------------------------------
+def new_state(n: int, device="cuda", stream=None):
+    """Allocate n stride_scan_state on the device and initialise them."""
+    torch = _torch()
+    st = torch.empty((max(n, 1), STATE_DTYPE.itemsize), dtype=torch.uint8, device=device)
+    stride_state_init(st, n, stream)
+    return st
+
+
+def new_turn_stats(n: int, device="cuda"):
+    torch = _torch()
+    return torch.zeros((max(n, 1), TURN_STATS_DTYPE.itemsize), dtype=torch.uint8, device=device)
+
+
+def state_to_numpy(st) -> np.ndarray:
+    return st.detach().cpu().numpy().reshape(-1).view(STATE_DTYPE)
+
+
+def turn_stats_to_numpy(ts) -> np.ndarray:
+    return ts.detach().cpu().numpy().reshape(-1).view(TURN_STATS_DTYPE)
+
+
+# ---------------------------------------------------------------------------
+# the C ABI, one function each
+# ---------------------------------------------------------------------------
+def stride_state_init(state, n: int, stream=None) -> None:
+    torch = _torch()
+    p = _dev(state, "state", torch.uint8, n * STATE_DTYPE.itemsize)
+    _check("stride_state_init", lib().stride_state_init(p, int(n), _stream(stream)))
+
+
+def stride_score_batch_workspace_size(window_rows: int) -> int:
+    return int(lib().stride_score_batch_workspace_size(int(window_rows)))
+
+
+def stride_score_batch(S, T, tokens, traj_row_off, turn_row_off, traj_turn_off, row_begin: int,
+                       row_end: int, stop_mode: int, lam, state, out: dict | None = None,
+                       turn_stats=None, dev_status=None, workspace=None, V: int | None = None,
+                       stream=None) -> None:
+    """Score global rows [row_begin, row_end) of a ragged trajectory layout.
+
+    S, T: [row_end-row_begin, ld] bf16/fp32 logits of those rows; tokens int32;
+    offsets int64/int64/int32 device tensors of the whole layout; lam a float
+    or a float32 [n_traj] tensor; state from :func:`new_state`; out a dict
+    of float32 [rows] tensors keyed by ROW_OUTPUT_KEYS; turn_stats from
+    :func:`new_turn_stats`; dev_status an int32 [1] tensor; workspace a uint8
+    tensor of at least stride_score_batch_workspace_size(rows) bytes (256-byte
+    aligned; torch's allocator returns such blocks)."""
+    torch = _torch()
+    dt, ld = _logits(S, T)
+    rows = int(row_end) - int(row_begin)
+    V = S.shape[1] if V is None else int(V)
+    n_traj = traj_row_off.numel() - 1
+    n_turns = turn_row_off.numel() - 1
+    lam_p, lam_all = _lambda(lam, n_traj)
+    ws_p = _dev(workspace, "workspace", torch.uint8, optional=True)  # size checked by the library
+    rc = lib().stride_score_batch(
+        S.data_ptr(), T.data_ptr(), dt, ld, V, _dev(tokens, "tokens", torch.int32, rows),
+        _dev(traj_row_off, "traj_row_off", torch.int64), _dev(turn_row_off, "turn_row_off", torch.int64),
+        _dev(traj_turn_off, "traj_turn_off", torch.int32), n_traj, n_turns, int(row_begin),
+        int(row_end), int(stop_mode), lam_p, lam_all,
+        _dev(state, "state", torch.uint8, n_traj * STATE_DTYPE.itemsize), _row_outputs(out, rows),
+        _dev(turn_stats, "turn_stats", torch.uint8, n_turns * TURN_STATS_DTYPE.itemsize, optional=True),
+        _dev(dev_status, "dev_status", torch.int32, 1, optional=True), ws_p,
+        0 if workspace is None else workspace.numel(), _stream(stream))
+    _check("stride_score_batch", rc)
+
+
+def stride_score_step(S, T, tokens, turn_end, stop_mode: int, lam, state, out: dict | None = None,
+                      stopped_now=None, turn_out=None, dev_status=None, V: int | None = None,
+                      stream=None) -> None:
+    """One decode step over B = S.shape[0] rollouts (see include/stride.h)."""
+    torch = _torch()
+    dt, ld = _logits(S, T)
+    B = S.shape[0]
+    V = S.shape[1] if V is None else int(V)
+    lam_p, lam_all = _lambda(lam, B)
+    rc = lib().stride_score_step(
+        S.data_ptr(), T.data_ptr(), dt, ld, V, _dev(tokens, "tokens", torch.int32, B),
+        _dev(turn_end, "turn_end", torch.uint8, B), B, int(stop_mode), lam_p, lam_all,
+        _dev(state, "state", torch.uint8, B * STATE_DTYPE.itemsize), _row_outputs(out, B),
+        _dev(stopped_now, "stopped_now", torch.uint8, B, optional=True),
+        _dev(turn_out, "turn_out", torch.uint8, B * TURN_STATS_DTYPE.itemsize, optional=True),
+        _dev(dev_status, "dev_status", torch.int32, 1, optional=True), _stream(stream))
+    _check("stride_score_step", rc)
+
+
+def stride_select_restart(turn_mean, n_turns, correct, alpha: float, k_star, k_max, stream=None) -> None:
+    """Restart choice (Eq. 6) over N records: turn_mean float32 [N, T_max],
+    n_turns int32 [N], correct uint8 [N, T_max] or None; outputs int32 [N]."""
+    torch = _torch()
+    if turn_mean.dim() != 2:
+        raise ValueError("turn_mean must be [N, T_max]")
+    N, T_max = turn_mean.shape
+    rc = lib().stride_select_restart(
+        _dev(turn_mean, "turn_mean", torch.float32, N * T_max), _dev(n_turns, "n_turns", torch.int32, N),
+        _dev(correct, "correct", torch.uint8, N * T_max, optional=True), float(alpha), N, T_max,
+        _dev(k_star, "k_star", torch.int32, N), _dev(k_max, "k_max", torch.int32, N), _stream(stream))
+    _check("stride_select_restart", rc)

@@ -1,0 +1,88 @@
+// stride_internal.h -- launch interfaces between the C-ABI layer and the
+// kernels.  Not installed; callers use include/stride.h.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stddef.h>
+#include <stdint.h>
+
+#include "stride.h"
+
+namespace stride {
+
+// One published scan element of the batch kernel's lookback (32 bytes).
+struct alignas(32) ScanSlot {
+  double c, st, sd, pad;
+};
+
+struct BatchParams {
+  const void* S;
+  const void* T;
+  int64_t ld;
+  int32_t V;
+  int32_t mode;
+  const int32_t* tokens;
+  const int64_t* traj_row_off;
+  const int64_t* turn_row_off;
+  const int32_t* traj_turn_off;
+  int32_t n_traj;
+  int32_t n_turns;
+  int64_t row_begin;
+  int64_t row_end;
+  int64_t n_rows;
+  const float* lambda;
+  float lambda_all;
+  stride_scan_state* state;
+  stride_row_outputs out;
+  stride_turn_stats* turn_stats;
+  int32_t* dev_status;
+  // workspace views
+  uint32_t* ticket;
+  uint32_t* flags;
+  ScanSlot* agg;
+  ScanSlot* incl;
+  uint64_t timeout_ns;
+};
+
+struct StepParams {
+  const void* S;
+  const void* T;
+  int64_t ld;
+  int32_t V;
+  int32_t mode;
+  const int32_t* tokens;
+  const uint8_t* turn_end;
+  int32_t B;
+  const float* lambda;
+  float lambda_all;
+  stride_scan_state* state;
+  stride_row_outputs out;
+  uint8_t* stopped_now;
+  stride_turn_stats* turn_out;
+  int32_t* dev_status;
+};
+
+struct SelectParams {
+  const float* turn_mean;
+  const int32_t* n_turns;
+  const uint8_t* correct;
+  float alpha;
+  int32_t N;
+  int32_t T_max;
+  int32_t* k_star;
+  int32_t* k_max;
+};
+
+// Workspace layout of stride_score_batch (all offsets 256-byte aligned).
+struct BatchWorkspaceLayout {
+  size_t ticket_off, flags_off, agg_off, incl_off, clear_bytes, total;
+};
+BatchWorkspaceLayout batch_workspace_layout(int64_t n_rows);
+
+// Launchers return a cudaError_t from the launch.
+cudaError_t launch_score_batch(const BatchParams& p, int dtype, bool vec, cudaStream_t stream);
+cudaError_t launch_score_step(const StepParams& p, int dtype, bool vec, cudaStream_t stream);
+cudaError_t launch_select_restart(const SelectParams& p, cudaStream_t stream);
+cudaError_t launch_state_init(stride_scan_state* state, int32_t n, cudaStream_t stream);
+
+}  // namespace stride

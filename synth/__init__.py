@@ -20,12 +20,47 @@ generated on the GPU with torch in fixed-size blocks, each block seeded from
 from __future__ import annotations
 
 import dataclasses
+import json
 import math
+from pathlib import Path
 
 import numpy as np
 
 V_QWEN3 = 151_936
 GEN_BLOCK = 512  # rows per independently seeded generation block
+
+# lambda of each ragged bf16 workload, written by tests/golden/calibrate_lambda.py
+CALIBRATION = Path(__file__).resolve().parents[1] / "tests" / "golden" / "lambda_calibration.json"
+# used only until a calibration exists (a round number near the expected value)
+PROVISIONAL_LAMBDA = {
+    "batch_scoring_64x8_v151936_bf16": -36.0,
+    "long_agentic_16x30_v151936_bf16": -170.0,
+    "multi_teacher_128x12_v151936_bf16": -55.0,
+}
+
+
+def load_calibration(name: str) -> dict | None:
+    if not CALIBRATION.exists():
+        return None
+    return json.loads(CALIBRATION.read_text()).get(name)
+
+
+def workload_lambda(name: str) -> float:
+    cal = load_calibration(name)
+    return float(np.float32(cal["lambda"] if cal else PROVISIONAL_LAMBDA[name]))
+
+
+def first_trajectories(lay: "Layout", max_rows: int) -> int:
+    """Number of leading trajectories whose rows fit in max_rows (at least 1)."""
+    n = int(np.searchsorted(lay.traj_row_off, lay.traj_row_off[0] + max_rows, side="right") - 1)
+    return max(1, min(n, lay.n_traj))
+
+
+def sub_layout(lay: "Layout", n_traj: int) -> "Layout":
+    """The layout of the first n_traj trajectories."""
+    k = int(lay.traj_turn_off[n_traj])
+    return Layout(lay.traj_row_off[: n_traj + 1].copy(), lay.turn_row_off[: k + 1].copy(),
+                  lay.traj_turn_off[: n_traj + 1].copy())
 
 
 # --------------------------------------------------------------------------
@@ -367,5 +402,6 @@ def describe_recipe() -> str:
 __all__ = [
     "V_QWEN3", "GEN_BLOCK", "Layout", "RowRecipe", "Workload", "bf16_bits_from_f32", "f32_from_bf16_bits",
     "layout_from_turn_lengths", "ragged_layout", "tiny_reference", "batch_scoring", "long_agentic",
-    "multi_teacher", "decode_steps", "generate_rows", "math",
+    "multi_teacher", "decode_steps", "generate_rows", "load_calibration", "workload_lambda",
+    "first_trajectories", "sub_layout",
 ]

@@ -148,6 +148,20 @@ def check_torch_log_softmax(orc):
     assert np.max(np.abs(o["logp_t"] - lt.numpy())) <= 1e-12
 
 
+def check_teacher_only(orc):
+    """S = None scores the teacher alone with the same results."""
+    rng = np.random.default_rng(16)
+    V = 500
+    S = (rng.standard_normal((5, V)) * 3).astype(np.float32)
+    T = (rng.standard_normal((5, V)) * 3).astype(np.float32)
+    y = rng.integers(0, V, 5).astype(np.int32)
+    a = orc.row_logprobs(S, T, y)
+    b = orc.row_logprobs(None, T, y)
+    assert np.array_equal(a["logp_t"], b["logp_t"]) and np.isnan(b["logp_s"]).all()
+    lt = np.array([math.log(math.fsum(math.exp(float(v)) for v in row)) for row in T])
+    assert np.max(np.abs(b["logp_t"] - (T[np.arange(5), y] - lt))) <= 1e-12
+
+
 def check_bf16_decode(orc):
     """bf16 bit patterns decode to the values IEEE-754 fixes."""
     cases = {0x3F80: 1.0, 0xC0A0: -5.0, 0x4049: 3.140625, 0x0001: 2.0 ** -133,
@@ -417,7 +431,7 @@ def check_select_bruteforce(orc):
 ALL_CHECKS = [
     check_uniform_closed_form, check_one_hot_closed_form, check_d_sign_and_operands,
     check_bruteforce_mpmath, check_normalisation, check_shift_invariance, check_torch_log_softmax,
-    check_bf16_decode, check_special_values, check_strided_rows,
+    check_teacher_only, check_bf16_decode, check_special_values, check_strided_rows,
     check_stop_rule_golden, check_prefix_buffer_offset, check_scan_invariants,
     check_traj_independence, check_per_trajectory_lambda, check_empty_turn_rejected,
     check_step_matches_batch, check_step_golden,

@@ -13,8 +13,10 @@ MUTANTS = [
     ("lse_drops_max", "return m + log(s);", "return log(s);"),
     ("d_sign", "jb->d[r] = ps - pt;", "jb->d[r] = pt - ps;"),
     ("teacher_uses_student_lse", "pt = xt - lt;", "pt = xt - ls;"),
-    ("gather_off_by_one", "xs = logit_at(jb->S, jb->dtype, jb->ld, r, y);",
-     "xs = logit_at(jb->S, jb->dtype, jb->ld, r, (y + 1) % jb->V);"),
+    ("gather_off_by_one", "xs = jb->S ? logit_at(jb->S, jb->dtype, jb->ld, r, y) : NAN;",
+     "xs = jb->S ? logit_at(jb->S, jb->dtype, jb->ld, r, (y + 1) % jb->V) : NAN;"),
+    ("teacher_gather_uses_student", "xt = logit_at(jb->T, jb->dtype, jb->ld, r, y);",
+     "xt = jb->S ? logit_at(jb->S, jb->dtype, jb->ld, r, y) : 0.0;"),
     ("bf16_shift", "((uint32_t)h) << 16", "((uint32_t)h) << 15"),
     ("max_skips_last", "for (int64_t j = 0; j < V; ++j) {\n    double x = logit_at(base, dtype, ld, r, j);\n    if (x > m) m = x;",
      "for (int64_t j = 0; j + 1 < V; ++j) {\n    double x = logit_at(base, dtype, ld, r, j);\n    if (x > m) m = x;"),
