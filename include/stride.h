@@ -71,7 +71,8 @@ typedef enum stride_status {
   STRIDE_ERR_UNSUPPORTED_DTYPE = 2,  /* dtype is not BF16 or F32 */
   STRIDE_ERR_WORKSPACE = 3,          /* workspace missing, too small or misaligned */
   STRIDE_ERR_CUDA = 4,               /* a CUDA runtime call or launch failed */
-  STRIDE_ERR_UNSUPPORTED_DEVICE = 5  /* current device is not compute capability 10.3 */
+  STRIDE_ERR_UNSUPPORTED_DEVICE = 5, /* current device is not compute capability 10.3 */
+  STRIDE_ERR_TOO_LARGE = 6           /* window larger than STRIDE_NOALLOC_MAX_ROWS (no-allocation entry point) */
 } stride_status;
 
 /* ---- device status bits (OR-ed into *dev_status) ----------------------- */
@@ -213,6 +214,39 @@ STRIDE_API int stride_score_step(const void* S, const void* T, int32_t dtype, in
 STRIDE_API int stride_select_restart(const float* turn_mean, const int32_t* n_turns, const uint8_t* correct,
                           float alpha, int32_t N, int32_t T_max, int32_t* k_star,
                           int32_t* k_max, void* stream);
+
+/* stride_score_batch for callers that cannot allocate device memory.
+ *
+ * The paper has no counterpart: this is a deployment variant of
+ * stride_score_batch.  Some callers cannot provide the scratch workspace,
+ * because the device memory is reserved up front by another allocator (a
+ * framework's caching allocator, a serving engine's cache pool) so that one
+ * more cudaMalloc fails or fragments it, because their path cannot take the
+ * implicit device synchronisation of cudaMalloc/cudaFree, or because they
+ * were handed only inputs and outputs.  This entry point takes the same
+ * arguments minus the workspace and uses a fixed scratch array that the
+ * library holds on every device that loads it (about 4.5 MB) until the
+ * process exits.  It allocates nothing.
+ *
+ * - Windows of more than STRIDE_NOALLOC_MAX_ROWS rows return
+ *   STRIDE_ERR_TOO_LARGE; nothing is launched.  Score longer inputs in
+ *   windows (the carried state makes that exact).
+ * - All calls on a device share the one scratch array, which keeps the last
+ *   call's contents; each call clears what must start at zero.  Calls that
+ *   overlap in time on the GPU race on it: order them on one stream.
+ * - The first call on a device looks up the array's device address
+ *   (cudaGetSymbolAddress, once per device); make that first call before any
+ *   stream capture. */
+#define STRIDE_NOALLOC_MAX_ROWS 65536
+STRIDE_API int stride_score_batch_noalloc(const void* S, const void* T, int32_t dtype, int64_t ld,
+                                          int64_t V, const int32_t* tokens,
+                                          const int64_t* traj_row_off, const int64_t* turn_row_off,
+                                          const int32_t* traj_turn_off, int32_t n_traj,
+                                          int32_t n_turns, int64_t row_begin, int64_t row_end,
+                                          int32_t stop_mode, const float* lambda, float lambda_all,
+                                          stride_scan_state* state, const stride_row_outputs* out,
+                                          stride_turn_stats* turn_stats, int32_t* dev_status,
+                                          void* stream);
 
 /* Human-readable name of a stride_status code (static string). */
 STRIDE_API const char* stride_status_string(int code);

@@ -28,12 +28,15 @@ __all__ = [
     "new_turn_stats", "state_to_numpy", "turn_stats_to_numpy", "stride_state_init",
     "stride_score_batch_workspace_size", "stride_score_batch", "stride_score_step",
     "stride_select_restart", "stride_status_string", "stride_abi_version", "ROW_OUTPUT_KEYS",
+    "stride_score_batch_noalloc", "NOALLOC_MAX_ROWS", "ERR_TOO_LARGE",
 ]
 
 DTYPE_BF16, DTYPE_F32 = 0, 1
 TURN_MEAN, TOKEN_SUM = 0, 1
 DEV_TOKEN_RANGE, DEV_BAD_LAYOUT, DEV_TIMEOUT = 0x1, 0x2, 0x4
 ROW_OUTPUT_KEYS = ("logp_s", "logp_t", "opd", "lse_s", "lse_t", "x_s", "x_t")
+NOALLOC_MAX_ROWS = 65536  # STRIDE_NOALLOC_MAX_ROWS
+ERR_TOO_LARGE = 6
 
 STATE_DTYPE = np.dtype([("cum", "<f8"), ("turn_sum_t", "<f8"), ("turn_sum_d", "<f8"),
                         ("rows_seen", "<i8"), ("stop_row", "<i8"), ("stop_turn", "<i4"),
@@ -74,10 +77,13 @@ def lib() -> ctypes.CDLL:
                                          P, P, P, P, P, sz, P]
         L.stride_score_step.argtypes = [P, P, i32, i64, i64, P, P, i32, i32, P, f32, P, P, P, P, P, P]
         L.stride_select_restart.argtypes = [P, P, P, f32, i32, i32, P, P, P]
+        L.stride_score_batch_noalloc.argtypes = [P, P, i32, i64, i64, P, P, P, P, i32, i32, i64, i64, i32,
+                                                 P, f32, P, P, P, P, P]
         L.stride_status_string.argtypes = [ctypes.c_int]
         L.stride_status_string.restype = ctypes.c_char_p
         L.stride_abi_version.restype = ctypes.c_int
-        for fn in ("stride_state_init", "stride_score_batch", "stride_score_step", "stride_select_restart"):
+        for fn in ("stride_state_init", "stride_score_batch", "stride_score_step", "stride_select_restart",
+                   "stride_score_batch_noalloc"):
             getattr(L, fn).restype = ctypes.c_int
         _LIB = L
     return _LIB
@@ -267,3 +273,28 @@ def stride_select_restart(turn_mean, n_turns, correct, alpha: float, k_star, k_m
         _dev(correct, "correct", torch.uint8, N * T_max, optional=True), float(alpha), N, T_max,
         _dev(k_star, "k_star", torch.int32, N), _dev(k_max, "k_max", torch.int32, N), _stream(stream))
     _check("stride_select_restart", rc)
+
+
+def stride_score_batch_noalloc(S, T, tokens, traj_row_off, turn_row_off, traj_turn_off, row_begin: int,
+                               row_end: int, stop_mode: int, lam, state, out: dict | None = None,
+                               turn_stats=None, dev_status=None, V: int | None = None, stream=None) -> None:
+    """stride_score_batch without a workspace argument, for callers that
+    cannot allocate device memory: the library's built-in scratch (at most
+    NOALLOC_MAX_ROWS rows per call) is used instead.  Calls that overlap on
+    the GPU race on that scratch; order them on one stream."""
+    torch = _torch()
+    dt, ld = _logits(S, T)
+    rows = int(row_end) - int(row_begin)
+    V = S.shape[1] if V is None else int(V)
+    n_traj = traj_row_off.numel() - 1
+    n_turns = turn_row_off.numel() - 1
+    lam_p, lam_all = _lambda(lam, n_traj)
+    rc = lib().stride_score_batch_noalloc(
+        S.data_ptr(), T.data_ptr(), dt, ld, V, _dev(tokens, "tokens", torch.int32, max(rows, 0)),
+        _dev(traj_row_off, "traj_row_off", torch.int64), _dev(turn_row_off, "turn_row_off", torch.int64),
+        _dev(traj_turn_off, "traj_turn_off", torch.int32), n_traj, n_turns, int(row_begin),
+        int(row_end), int(stop_mode), lam_p, lam_all,
+        _dev(state, "state", torch.uint8, n_traj * STATE_DTYPE.itemsize), _row_outputs(out, max(rows, 0)),
+        _dev(turn_stats, "turn_stats", torch.uint8, n_turns * TURN_STATS_DTYPE.itemsize, optional=True),
+        _dev(dev_status, "dev_status", torch.int32, 1, optional=True), _stream(stream))
+    _check("stride_score_batch_noalloc", rc)

@@ -67,6 +67,7 @@ const char* stride_status_string(int code) {
     case STRIDE_ERR_WORKSPACE: return "STRIDE_ERR_WORKSPACE: workspace missing, too small or not 256-byte aligned";
     case STRIDE_ERR_CUDA: return "STRIDE_ERR_CUDA: a CUDA runtime call or kernel launch failed";
     case STRIDE_ERR_UNSUPPORTED_DEVICE: return "STRIDE_ERR_UNSUPPORTED_DEVICE: the current device is not sm_103 (GB300)";
+    case STRIDE_ERR_TOO_LARGE: return "STRIDE_ERR_TOO_LARGE: window exceeds STRIDE_NOALLOC_MAX_ROWS rows of the built-in scratch";
     default: return "unknown stride status";
   }
 }
