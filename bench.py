@@ -61,7 +61,7 @@ def kernel_traffic_record() -> tuple[float | None, str]:
     summary, valid only while the kernel source is unchanged."""
     src = ROOT / "paper_2609_14636_gb300" / "csrc"
     h = hashlib.sha256()
-    for f in ("score_batch.cu", "stride_device.cuh"):
+    for f in ("score_batch_stream.cu", "row_scan.cuh", "stride_device.cuh"):
         h.update((src / f).read_bytes())
     digest = h.hexdigest()[:16]
     rec = ROOT / "profiles" / "score_batch_traffic.txt"
@@ -344,7 +344,7 @@ def main() -> None:
     roofline = {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s", "frac": achieved / peak,
                 "traffic": None if dram_per_row is None else dram_per_row * R,
                 "algorithmic_bytes_per_launch": bpr * R, "kernel_ms_mean": k_avg,
-                "kernel_ms_min": min(k_ms), "kernel": "score_batch_kernel<bf16,vec>",
+                "kernel_ms_min": min(k_ms), "kernel": "score_batch_stream_kernel<bf16>",
                 "peak_source": "MEASURED_PEAKS.json hbm_gbs (of measured)" if "hbm_gbs" in peaks else "fallback 6.8 TB/s"}
 
     # ---- end to end from pinned host buffers ------------------------------

@@ -81,6 +81,7 @@ BatchWorkspaceLayout batch_workspace_layout(int64_t n_rows);
 
 // Launchers return a cudaError_t from the launch.
 cudaError_t launch_score_batch(const BatchParams& p, int dtype, bool vec, cudaStream_t stream);
+cudaError_t launch_score_batch_stream(const BatchParams& p, int dtype, cudaStream_t stream);
 cudaError_t launch_score_step(const StepParams& p, int dtype, bool vec, cudaStream_t stream);
 cudaError_t launch_select_restart(const SelectParams& p, cudaStream_t stream);
 cudaError_t launch_state_init(stride_scan_state* state, int32_t n, cudaStream_t stream);
