@@ -240,12 +240,17 @@ def load_lambda(w) -> np.ndarray:
     return np.full(w.layout.n_traj, np.float32(synth.workload_lambda(w.name)), np.float32)
 
 
+WORKLOADS = ("batch_scoring", "long_agentic", "multi_teacher", "decode_step", "select")
+
+
 def main() -> None:
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--steps", type=int, default=100)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--workload", choices=WORKLOADS, default="batch_scoring",
+                    help="batch_scoring is the headline; the others measure the remaining rows of the path")
     ap.add_argument("--cpu-budget", type=float, default=12.0, help="seconds of oracle time for cpu_baseline")
     ap.add_argument("--e2e-rows", type=int, default=8192)
     ap.add_argument("--max-rows", type=int, default=0,
@@ -254,7 +259,15 @@ def main() -> None:
     if args.impl == "reference":
         run_reference(args)
         return
+    if args.workload == "decode_step":
+        run_decode(args)
+    elif args.workload == "select":
+        run_select(args)
+    else:
+        run_batch(args)
 
+
+def _setup_rank():
     import torch
 
     ws, rank, local = dist_env()
@@ -263,12 +276,30 @@ def main() -> None:
 
         dist.init_process_group("nccl")
     torch.cuda.set_device(local)
-    dev = torch.device("cuda", local)
+    return ws, rank, local, torch.device("cuda", local)
+
+
+def _common_line(args, ws, ms_step, value, unit=UNIT, metric=METRIC, dtype="bf16"):
+    return {"metric": metric, "value": value, "unit": unit, "n_gpus": ws, "steps": args.steps,
+            "warmup": max(3, args.warmup), "ms_per_step": ms_step, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": dtype, "data": "synthetic"}
+
+
+def run_batch(args) -> None:
+    """Ragged batch scoring: the headline workload (all rows in one window), or
+    the long-agentic / multi-teacher workloads resident in HBM and scored in
+    their 16,384-row windows with the carried state."""
+    import torch
+
+    ws, rank, local, dev = _setup_rank()
+    if ws > 1:
+        import torch.distributed as dist
 
     import paper_2609_14636_gb300 as stride
     import synth
 
-    w = synth.batch_scoring()
+    w = {"batch_scoring": synth.batch_scoring, "long_agentic": synth.long_agentic,
+         "multi_teacher": synth.multi_teacher}[args.workload]()
     lay = w.layout
     if args.max_rows > 0:
         lay = synth.sub_layout(lay, synth.first_trajectories(lay, args.max_rows))
@@ -292,15 +323,19 @@ def main() -> None:
     ts = stride.new_turn_stats(lay.n_turns, dev)
     out = {k: torch.empty(R, dtype=torch.float32, device=dev) for k in ("logp_s", "logp_t", "opd")}
     status = torch.zeros(1, dtype=torch.int32, device=dev)
-    wsb = torch.empty(stride.stride_score_batch_workspace_size(R), dtype=torch.uint8, device=dev)
+    chunk = int(w.extra.get("chunk_rows", R))
+    windows = [(a, min(R, a + chunk)) for a in range(0, R, chunk)]
+    wsb = torch.empty(stride.stride_score_batch_workspace_size(min(chunk, R)), dtype=torch.uint8, device=dev)
     stream = torch.cuda.current_stream()
 
     def step(ev=None):
         stride.stride_state_init(st, lay.n_traj, stream)
         if ev is not None:
             ev[0].record(stream)
-        stride.stride_score_batch(S, T, tok, *offs, 0, R, stride.TURN_MEAN, lam_d, st, out=out, turn_stats=ts,
-                                  dev_status=status, workspace=wsb, stream=stream)
+        for a, b in windows:
+            stride.stride_score_batch(S[a:b], T[a:b], tok[a:b], *offs, a, b, stride.TURN_MEAN, lam_d, st,
+                                      out={k: v[a:b] for k, v in out.items()}, turn_stats=ts,
+                                      dev_status=status, workspace=wsb, stream=stream)
         if ev is not None:
             ev[1].record(stream)
 
@@ -338,7 +373,7 @@ def main() -> None:
     peaks = measured_peaks()
     peak = peaks.get("hbm_gbs", 6800.0)
     bpr = algorithmic_bytes_per_row(V)
-    k_avg = statistics.mean(k_ms)
+    k_avg = statistics.mean(k_ms)  # all windows of one step
     achieved = bpr * R / (k_avg * 1e-3) / 1e9
     dram_per_row, digest = kernel_traffic_record()
     roofline = {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s", "frac": achieved / peak,
@@ -371,13 +406,17 @@ def main() -> None:
         ets = stride.new_turn_stats(n_tu, dev)
         eout = {k: v[:Re] for k, v in out.items()}
 
+        ewin = [(a, min(Re, a + chunk)) for a in range(0, Re, chunk)]
+
         def e2e_step():
             dS.copy_(hS, non_blocking=True)
             dT.copy_(hT, non_blocking=True)
             dk.copy_(hk, non_blocking=True)
             stride.stride_state_init(est, n_tr, stream)
-            stride.stride_score_batch(dS, dT, dk, *eoffs, 0, Re, stride.TURN_MEAN, lam_d[:n_tr], est, out=eout,
-                                      turn_stats=ets, dev_status=status, workspace=wsb, stream=stream)
+            for a, b in ewin:
+                stride.stride_score_batch(dS[a:b], dT[a:b], dk[a:b], *eoffs, a, b, stride.TURN_MEAN, lam_d[:n_tr],
+                                          est, out={k: v[a:b] for k, v in eout.items()}, turn_stats=ets,
+                                          dev_status=status, workspace=wsb, stream=stream)
             for k in hout:
                 hout[k].copy_(eout[k], non_blocking=True)
             hst.copy_(est[:n_tr], non_blocking=True)
@@ -409,24 +448,171 @@ def main() -> None:
 
     if rank == 0:
         clocks = clk.summary()
-        line = {
-            "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws, "steps": args.steps,
-            "warmup": max(3, args.warmup), "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak",
-            "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        line = _common_line(args, ws, ms_step, value)
+        line.update({
             "config": {"workload": w.name if args.max_rows <= 0 else f"{w.name} (first {lay.n_traj} trajectories)",
+                       "windows": len(windows), "window_rows": chunk,
                        "trajectories": lay.n_traj, "turns": lay.n_turns, "rows": R,
                        "vocab": V, "logits": "bf16 student + bf16 teacher, resident in HBM",
                        "bytes_resident": 2 * R * V * 2, "stop_mode": "turn_mean",
                        "lambda": float(lam[0]), "early_stop_fraction": early_frac,
                        "l2": f"inputs ({2 * R * V * 2 / 1e9:.1f} GB) larger than L2 (129 MB): no flush",
+                       "lambda_source": "tests/golden/lambda_calibration.json (oracle, 40% quantile)",
                        "parallelism": f"replicas x{ws}" if ws > 1 else "single GPU",
                        "generation_s": t_gen},
             "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e, "clocks": clocks,
-            "gpu_launches": 2 * args.steps,
-        }
+            "gpu_launches": (1 + len(windows)) * args.steps,
+        })
         print(json.dumps(line), flush=True)
     if ws > 1:
         dist.destroy_process_group()
+
+
+def _graph(fn):
+    """Capture fn() (a sequence of library calls on the current stream) in a
+    CUDA graph."""
+    import torch
+
+    g = torch.cuda.CUDAGraph()
+    s = torch.cuda.Stream()
+    s.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(s):
+        fn()  # warm: first calls on a device do their one-time set-up here
+    torch.cuda.current_stream().wait_stream(s)
+    torch.cuda.synchronize()
+    with torch.cuda.graph(g):
+        fn()
+    torch.cuda.synchronize()
+    return g
+
+
+def run_decode(args) -> None:
+    """Decode steps: B = 256 rollouts x 4,096 steps of stride_score_step, a
+    ring of 16 distinct [256, V] step slabs (more bytes than L2), turn ends
+    every U{96..768} steps, stopped rollouts masked; the 4,097 launches of a
+    sweep are replayed as one CUDA graph.  Also a 64-step graph with no stop
+    (lambda = -inf), which shows the kernel at full activity."""
+    import torch
+
+    ws, rank, local, dev = _setup_rank()
+    import paper_2609_14636_gb300 as stride
+    import synth
+
+    w = synth.decode_steps()
+    B, ring, n_steps = w["B"], w["ring"], w["steps"]
+    V = w["recipe"].V
+    S, T, tok = synth.generate_rows(w["recipe"], 0, ring * B, device=dev)
+    te = torch.from_numpy(w["turn_end"]).to(dev)
+    st = stride.new_state(B, dev)
+    out = {k: torch.empty(B, dtype=torch.float32, device=dev) for k in ("logp_s", "logp_t", "opd")}
+    sn = torch.empty(B, dtype=torch.uint8, device=dev)
+    tout = torch.empty((B, 32), dtype=torch.uint8, device=dev)
+    status = torch.zeros(1, dtype=torch.int32, device=dev)
+
+    def sweep(lam, steps):
+        stride.stride_state_init(st, B)
+        for i in range(steps):
+            j = i % ring
+            stride.stride_score_step(S[j * B:(j + 1) * B], T[j * B:(j + 1) * B], tok[j * B:(j + 1) * B], te[i],
+                                     stride.TURN_MEAN, lam, st, out=out, stopped_now=sn, turn_out=tout,
+                                     dev_status=status)
+
+    g_full = _graph(lambda: sweep(float("-inf"), 64))
+    g_run = _graph(lambda: sweep(w["lam_turn"], n_steps))
+    stream = torch.cuda.current_stream()
+    reps = max(1, min(args.steps, 10))
+    for _ in range(max(3, args.warmup)):
+        g_full.replay()
+    g_run.replay()
+    torch.cuda.synchronize()
+    if int(status.item()) != 0:
+        raise RuntimeError(f"device status {int(status.item())}")
+    scored = int(stride.state_to_numpy(st)["rows_seen"][:B].sum())
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with ClockSampler(local) as clk:
+        time.sleep(0.25)
+        a.record(stream)
+        for _ in range(reps):
+            g_run.replay()
+        b.record(stream)
+        torch.cuda.synchronize()
+        ms_sweep = a.elapsed_time(b) / reps
+        a.record(stream)
+        for _ in range(20):
+            g_full.replay()
+        b.record(stream)
+        torch.cuda.synchronize()
+        ms_full = a.elapsed_time(b) / 20
+        time.sleep(0.05)
+    ms_sweep = max_over_ranks(ms_sweep, dev)
+    bpr = algorithmic_bytes_per_row(V)
+    peak = measured_peaks().get("hbm_gbs", 6800.0)
+    us_step_full = 1e3 * ms_full / 64
+    full_gbs = B * bpr / (us_step_full * 1e-6) / 1e9
+    value = ws * scored / (ms_sweep * 1e-3)
+    if rank == 0:
+        line = _common_line(args, ws, ms_sweep, value)
+        line.update({
+            "config": {"workload": w["name"], "rollouts": B, "decode_steps": n_steps, "ring_slabs": ring,
+                       "vocab": V, "stop_mode": "turn_mean", "lambda": w["lam_turn"],
+                       "tokens_scored_per_sweep": scored, "graph": "one CUDA graph per 4,097-launch sweep",
+                       "l2": f"ring of {ring} slabs = {2 * ring * B * V * 2 / 1e9:.2f} GB > L2: no flush"},
+            "roofline": {"bound": "hbm", "achieved": full_gbs, "peak": peak, "unit": "GB/s", "frac": full_gbs / peak,
+                         "traffic": None, "kernel": "score_step_kernel<bf16,vec> (4-CTA clusters)",
+                         "us_per_step_all_active": us_step_full,
+                         "sweep_gbs_incl_masked_steps": scored * bpr / (ms_sweep * 1e-3) / 1e9,
+                         "peak_source": "MEASURED_PEAKS.json hbm_gbs (of measured)"},
+            "clocks": clk.summary(), "gpu_launches": reps * (n_steps + 1) + 20 * 65,
+        })
+        print(json.dumps(line), flush=True)
+
+
+def run_select(args) -> None:
+    """Restart choice over the 10,000-record prefix buffer (12 turns, masks
+    Bernoulli(0.5), alpha = -6.0): one launch per call, 200 calls per graph."""
+    import torch
+
+    ws, rank, local, dev = _setup_rank()
+    import paper_2609_14636_gb300 as stride
+    import synth
+
+    w = synth.multi_teacher()
+    means = torch.from_numpy(w.extra["buffer_means"]).to(dev)
+    nt = torch.from_numpy(w.extra["buffer_n_turns"]).to(dev)
+    mask = torch.from_numpy(w.extra["buffer_masks"]["p50"]).to(dev)
+    N, T_max = means.shape
+    ks = torch.empty(N, dtype=torch.int32, device=dev)
+    km = torch.empty(N, dtype=torch.int32, device=dev)
+    calls = 200
+    g = _graph(lambda: [stride.stride_select_restart(means, nt, mask, -6.0, ks, km) for _ in range(calls)])
+    stream = torch.cuda.current_stream()
+    for _ in range(max(3, args.warmup)):
+        g.replay()
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    reps = max(1, min(args.steps, 50))
+    with ClockSampler(local) as clk:
+        time.sleep(0.25)
+        a.record(stream)
+        for _ in range(reps):
+            g.replay()
+        b.record(stream)
+        torch.cuda.synchronize()
+        time.sleep(0.05)
+    us_call = 1e3 * a.elapsed_time(b) / (reps * calls)
+    us_call = max_over_ranks(us_call, dev)
+    bytes_call = N * T_max * 5 + N * 12
+    if rank == 0:
+        line = _common_line(args, ws, us_call / 1e3, ws * N / (us_call * 1e-6), unit="records/s",
+                            metric="restart choices/sec (10,000 x 12 records)", dtype="f32")
+        line.update({
+            "config": {"workload": "prefix_buffer_select_10000x12", "records": N, "turns": T_max,
+                       "mask": "Bernoulli(0.5)", "alpha": -6.0, "graph": f"{calls} launches per CUDA graph"},
+            "roofline": {"bound": "latency", "achieved": bytes_call / (us_call * 1e-6) / 1e9, "peak": None,
+                         "unit": "GB/s", "frac": None, "traffic": None, "us_per_call": us_call,
+                         "kernel": "select_restart_kernel (one warp per record)"},
+            "clocks": clk.summary(), "gpu_launches": reps * calls,
+        })
+        print(json.dumps(line), flush=True)
 
 
 if __name__ == "__main__":

@@ -44,15 +44,20 @@ def up_to_date() -> bool:
     return all(p.stat().st_mtime <= t for p in _deps())
 
 
-def build(force: bool = False, verbose: bool = False) -> Path:
-    if not force and up_to_date():
+def build(force: bool = False, verbose: bool = False, defines: tuple = (), lib: Path | None = None,
+          build_dir: Path | None = None) -> Path:
+    """Compile and link.  `defines` adds -D flags (tuning knobs of the
+    kernels); `lib`/`build_dir` redirect the output (default: in-tree)."""
+    out_lib = LIB if lib is None else Path(lib)
+    bdir = BUILD if build_dir is None else Path(build_dir)
+    if not force and lib is None and not defines and up_to_date():
         return LIB
-    BUILD.mkdir(exist_ok=True)
+    bdir.mkdir(parents=True, exist_ok=True)
     objs = []
 
     def compile_one(src: Path) -> tuple[Path, str]:
-        obj = BUILD / (src.stem + ".o")
-        cmd = [nvcc(), *ARCH, *NVCC_FLAGS, "-c", str(src), "-o", str(obj)]
+        obj = bdir / (src.stem + ".o")
+        cmd = [nvcc(), *ARCH, *NVCC_FLAGS, *[f"-D{d}" for d in defines], "-c", str(src), "-o", str(obj)]
         r = subprocess.run(cmd, capture_output=True, text=True)
         if r.returncode != 0:
             raise RuntimeError(f"nvcc failed for {src.name}:\n{r.stdout}\n{r.stderr}")
@@ -64,16 +69,16 @@ def build(force: bool = False, verbose: bool = False) -> Path:
     for obj, err in results:
         objs.append(obj)
         log.append(err)
-    (BUILD / "ptxas.log").write_text("\n".join(log))
-    tmp = LIB.with_name(LIB.name + f".tmp{os.getpid()}")
+    (bdir / "ptxas.log").write_text("\n".join(log))
+    tmp = out_lib.with_name(out_lib.name + f".tmp{os.getpid()}")
     cmd = [nvcc(), *ARCH, "-shared", "-cudart", "shared", "-o", str(tmp), *map(str, objs)]
     r = subprocess.run(cmd, capture_output=True, text=True)
     if r.returncode != 0:
         raise RuntimeError(f"link failed:\n{r.stdout}\n{r.stderr}")
-    os.replace(tmp, LIB)
+    os.replace(tmp, out_lib)
     if verbose:
         print("\n".join(log))
-    return LIB
+    return out_lib
 
 
 if __name__ == "__main__":

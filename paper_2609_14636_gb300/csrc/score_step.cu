@@ -10,6 +10,16 @@
 // carried state (open-turn sums, turn close with Eq. 4, stop test of Eq. 5 or
 // Sec. 5.5).  Rollouts whose state says stopped exit before reading a byte.
 // No workspace, no atomics, no spin-waits: the cluster barrier is hardware.
+//
+// Launch shape (chosen by a sweep of CTA size x cluster size x unroll on
+// GB300, B = 256, V = 151,936): 128-thread CTAs, 4 per cluster, at most 64
+// registers so 8 fit per SM, so a 256-rollout step is one wave of 1,024
+// CTAs (27.5 us per step; 8-CTA clusters of 256 threads took 44.7 us, 128-
+// thread CTAs in 8-CTA clusters 35.9 us).  Steps are launched with programmatic
+// dependent launch: a step's CTAs may be scheduled while the previous
+// kernel on the stream finishes, and each waits (griddepcontrol.wait) for
+// that kernel's completion before its first global read, so the caller's
+// inputs and the carried state are always complete when read.
 #include <cooperative_groups.h>
 #include <math.h>
 
@@ -21,13 +31,26 @@ namespace cg = cooperative_groups;
 
 namespace stride {
 
-constexpr int kStepThreads = 256;
+#ifndef STRIDE_STEP_THREADS
+#define STRIDE_STEP_THREADS 128
+#endif
+#ifndef STRIDE_STEP_CLUSTER
+#define STRIDE_STEP_CLUSTER 4
+#endif
+#ifndef STRIDE_STEP_UNROLL
+#define STRIDE_STEP_UNROLL 4
+#endif
+#ifndef STRIDE_STEP_MIN_BLOCKS
+#define STRIDE_STEP_MIN_BLOCKS 8
+#endif
+
+constexpr int kStepThreads = STRIDE_STEP_THREADS;
 constexpr int kStepWarps = kStepThreads / 32;
-constexpr int kStepCluster = 8;
-constexpr int kStepUnroll = 4;
+constexpr int kStepCluster = STRIDE_STEP_CLUSTER;
+constexpr int kStepUnroll = STRIDE_STEP_UNROLL;
 
 template <typename LT, bool VEC>
-__global__ void __cluster_dims__(kStepCluster, 1, 1) __launch_bounds__(kStepThreads)
+__global__ void __cluster_dims__(kStepCluster, 1, 1) __launch_bounds__(kStepThreads, STRIDE_STEP_MIN_BLOCKS)
     score_step_kernel(const StepParams p) {
   __shared__ float s_red[4][kStepWarps];
   __shared__ float s_part[4];
@@ -39,6 +62,8 @@ __global__ void __cluster_dims__(kStepCluster, 1, 1) __launch_bounds__(kStepThre
   const int warp = tid >> 5;
   stride_scan_state* sp = p.state + b;
   const float nan = __int_as_float(0x7fc00000);
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 
   // Every CTA of the cluster reads the flag before the first cluster barrier
   // and rank 0 writes it only after that barrier, so all agree.
@@ -183,19 +208,28 @@ __global__ void __cluster_dims__(kStepCluster, 1, 1) __launch_bounds__(kStepThre
   cluster.sync();  // peers keep their shared memory until rank 0 has read it
 }
 
+template <typename LT, bool VEC>
+static cudaError_t launch_step_pdl(const StepParams& p, cudaStream_t stream) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)p.B * kStepCluster);
+  cfg.blockDim = dim3(kStepThreads);
+  cfg.dynamicSmemBytes = 0;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, score_step_kernel<LT, VEC>, p);
+}
+
 cudaError_t launch_score_step(const StepParams& p, int dtype, bool vec, cudaStream_t stream) {
-  const dim3 grid((unsigned)p.B * kStepCluster), block(kStepThreads);
-  if (dtype == STRIDE_DTYPE_BF16) {
-    if (vec)
-      score_step_kernel<__nv_bfloat16, true><<<grid, block, 0, stream>>>(p);
-    else
-      score_step_kernel<__nv_bfloat16, false><<<grid, block, 0, stream>>>(p);
-  } else {
-    if (vec)
-      score_step_kernel<float, true><<<grid, block, 0, stream>>>(p);
-    else
-      score_step_kernel<float, false><<<grid, block, 0, stream>>>(p);
-  }
+  cudaError_t e;
+  if (dtype == STRIDE_DTYPE_BF16)
+    e = vec ? launch_step_pdl<__nv_bfloat16, true>(p, stream) : launch_step_pdl<__nv_bfloat16, false>(p, stream);
+  else
+    e = vec ? launch_step_pdl<float, true>(p, stream) : launch_step_pdl<float, false>(p, stream);
+  if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }
 
