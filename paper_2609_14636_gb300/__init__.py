@@ -77,6 +77,8 @@ def lib() -> ctypes.CDLL:
                                          P, P, P, P, P, sz, P]
         L.stride_score_step.argtypes = [P, P, i32, i64, i64, P, P, i32, i32, P, f32, P, P, P, P, P, P]
         L.stride_select_restart.argtypes = [P, P, P, f32, i32, i32, P, P, P]
+        L.stride_selftest_bounded_wait.argtypes = [i32, ctypes.c_uint64, P, P, sz, P]
+        L.stride_selftest_bounded_wait.restype = ctypes.c_int
         L.stride_score_batch_noalloc.argtypes = [P, P, i32, i64, i64, P, P, P, P, i32, i32, i64, i64, i32,
                                                  P, f32, P, P, P, P, P]
         L.stride_status_string.argtypes = [ctypes.c_int]
@@ -273,6 +275,18 @@ def stride_select_restart(turn_mean, n_turns, correct, alpha: float, k_star, k_m
         _dev(correct, "correct", torch.uint8, N * T_max, optional=True), float(alpha), N, T_max,
         _dev(k_star, "k_star", torch.int32, N), _dev(k_max, "k_max", torch.int32, N), _stream(stream))
     _check("stride_select_restart", rc)
+
+
+SELFTEST_LOOKBACK, SELFTEST_MBARRIER = 0, 1
+
+
+def stride_selftest_bounded_wait(which: int, timeout_ns: int, dev_status, workspace, stream=None) -> None:
+    """Run one of the library's bounded device waits on a flag nothing sets
+    (include/stride_selftest.h); the kernel ORs DEV_TIMEOUT into dev_status."""
+    torch = _torch()
+    rc = lib().stride_selftest_bounded_wait(int(which), int(timeout_ns), _dev(dev_status, "dev_status", torch.int32, 1),
+                                            _dev(workspace, "workspace", torch.uint8), workspace.numel(), _stream(stream))
+    _check("stride_selftest_bounded_wait", rc)
 
 
 def stride_score_batch_noalloc(S, T, tokens, traj_row_off, turn_row_off, traj_turn_off, row_begin: int,

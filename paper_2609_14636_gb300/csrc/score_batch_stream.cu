@@ -36,6 +36,7 @@
 // issuing, waits (bounded) for the copies it has in flight, and returns.
 #include <math.h>
 
+#include "mbarrier.cuh"
 #include "row_scan.cuh"
 #include "stride.h"
 #include "stride_device.cuh"
@@ -46,6 +47,9 @@
 #endif
 #ifndef STRIDE_BULK_CHUNK
 #define STRIDE_BULK_CHUNK 16384
+#endif
+#ifndef STRIDE_BULK_EVICT_FIRST
+#define STRIDE_BULK_EVICT_FIRST 1
 #endif
 
 namespace stride {
@@ -83,56 +87,6 @@ struct alignas(128) StreamShared {
 
 constexpr size_t kStreamHeader = (sizeof(StreamShared) + 127) & ~size_t(127);
 constexpr size_t kStreamSmem = kStreamHeader + 2 * (size_t)kStages * kChunk;
-
-__device__ __forceinline__ uint32_t smem_u32(const void* p) {
-  return (uint32_t)__cvta_generic_to_shared(p);
-}
-
-__device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
-  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count) : "memory");
-}
-
-__device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
-  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
-}
-
-__device__ __forceinline__ void mbar_arrive_expect_tx(uint64_t* bar, uint32_t bytes) {
-  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)), "r"(bytes)
-               : "memory");
-}
-
-__device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
-  uint32_t ok;
-  asm volatile(
-      "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n"
-      " selp.u32 %0, 1, 0, p;\n}"
-      : "=r"(ok)
-      : "r"(smem_u32(bar)), "r"(parity)
-      : "memory");
-  return ok != 0;
-}
-
-// Waits for the completion of the phase with the given parity; false once
-// timeout_ns has passed or another warp of the CTA has aborted.
-__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, uint64_t timeout_ns,
-                                          volatile int32_t* abort) {
-  if (mbar_try_wait(bar, parity)) return true;
-  const uint64_t t0 = globaltimer_ns();
-  while (true) {
-    if (mbar_try_wait(bar, parity)) return true;
-    if (*abort) return false;
-    if (globaltimer_ns() - t0 > timeout_ns) return false;
-  }
-}
-
-__device__ __forceinline__ void bulk_g2s(void* dst, const void* src, uint32_t bytes, uint64_t* bar,
-                                         uint64_t policy) {
-  asm volatile(
-      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint"
-      " [%0], [%1], %2, [%3], %4;" ::"r"(smem_u32(dst)),
-      "l"(src), "r"(bytes), "r"(smem_u32(bar)), "l"(policy)
-      : "memory");
-}
 
 __device__ __forceinline__ void raise_abort(StreamShared& sh, const BatchParams& p) {
   *reinterpret_cast<volatile int32_t*>(&sh.abort) = 1;
@@ -178,7 +132,11 @@ __global__ void __launch_bounds__(kStreamThreads, 1) score_batch_stream_kernel(c
     // ------------------------------------------------------------ producer
     if (lane == 0) {
       uint64_t policy;
+#if STRIDE_BULK_EVICT_FIRST
       asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(policy));
+#else
+      asm volatile("createpolicy.fractional.L2::evict_normal.b64 %0, 1.0;" : "=l"(policy));
+#endif
       uint32_t it = 0;  // stages issued
       int64_t seq = 0;  // rows started by this CTA
       bool ok = true;

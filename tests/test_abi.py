@@ -11,7 +11,7 @@ ROOT = Path(__file__).resolve().parents[1]
 
 
 def declared_symbols():
-    src = (ROOT / "include" / "stride.h").read_text()
+    src = "\n".join(p.read_text() for p in sorted((ROOT / "include").glob("*.h")))
     return sorted(set(re.findall(r"STRIDE_API\s+[\w\s\*]+?\b(stride_\w+)\s*\(", src)))
 
 
@@ -46,6 +46,6 @@ def test_host_only_calls():
 def test_header_compiles_as_c():
     pytest.importorskip("subprocess")
     r = subprocess.run(["gcc", "-std=c99", "-Wall", "-Werror", "-fsyntax-only", "-x", "c", "-I", str(ROOT / "include"), "-"],
-                       input='#include "stride.h"\nint main(void){return sizeof(stride_scan_state)==56 && sizeof(stride_turn_stats)==32 ? 0 : 1;}\n',
+                       input='#include "stride.h"\n#include "stride_selftest.h"\nint main(void){return sizeof(stride_scan_state)==56 && sizeof(stride_turn_stats)==32 ? 0 : 1;}\n',
                        capture_output=True, text=True)
     assert r.returncode == 0, r.stderr
