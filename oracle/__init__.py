@@ -58,9 +58,9 @@ class OracleLib:
         i64, i32, ci = ctypes.c_int64, ctypes.c_int32, ctypes.c_int
         lib.oracle_row_logprobs.argtypes = [P, P, ci, i64, i64, P, i64, P, P, P, P, P, P, P, ci]
         lib.oracle_row_logprobs.restype = ci
-        lib.oracle_scan_batch.argtypes = [P, P, P, P, P, i32, ci, P, P, P, P, P, P, P, P, P, P, P]
+        lib.oracle_scan_batch.argtypes = [P, P, P, P, P, P, i32, ci, P, P, P, P, P, P, P, P, P, P, P, P, P, P, P]
         lib.oracle_scan_batch.restype = ci
-        lib.oracle_step_update.argtypes = [P, P, P, i32, ci, P, P, P, P, P, P, P, P, P, P, P]
+        lib.oracle_step_update.argtypes = [P, P, P, i32, ci, P, P, P, P, P, P, P, P, P, P, P, P]
         lib.oracle_step_update.restype = ci
         lib.oracle_select_restart.argtypes = [P, P, P, ctypes.c_float, i32, i32, P, P]
         lib.oracle_select_restart.restype = ci
@@ -105,13 +105,15 @@ class OracleLib:
 
     # ---- Eq. 4 / Eq. 5 / Sec. 5.5: batch scan ------------------------------
     def scan_batch(self, logp_t, d, traj_row_off, turn_row_off, traj_turn_off, mode: int, lam,
-                   cum_in=None) -> dict:
-        """Turn means and the stop rule over ragged trajectories.
+                   cum_in=None, logp_s=None) -> dict:
+        """Turn means, the stop rule, the OPD loss on retained tokens (needs
+        logp_s) and the within-turn decile profile over ragged trajectories.
 
         ``lam`` is a scalar or a per-trajectory array.  Row arrays are indexed
         from ``traj_row_off[0]``."""
         logp_t = np.ascontiguousarray(logp_t, np.float64)
         d = None if d is None else np.ascontiguousarray(d, np.float64)
+        ls = None if logp_s is None else np.ascontiguousarray(logp_s, np.float64)
         tro = np.ascontiguousarray(traj_row_off, np.int64)
         uro = np.ascontiguousarray(turn_row_off, np.int64)
         tto = np.ascontiguousarray(traj_turn_off, np.int32)
@@ -120,17 +122,21 @@ class OracleLib:
         lam_a = np.ascontiguousarray(np.broadcast_to(np.asarray(lam, np.float64), (n_traj,)))
         cin = None if cum_in is None else np.ascontiguousarray(cum_in, np.float64)
         out = dict(
-            turn_sum_t=np.empty(n_turns), turn_sum_d=np.empty(n_turns), turn_mean=np.empty(n_turns),
-            turn_n=np.empty(n_turns, np.int64), turn_cum=np.empty(n_turns),
+            turn_sum_t=np.empty(n_turns), turn_sum_d=np.empty(n_turns), turn_sum_l=np.empty(n_turns),
+            turn_mean=np.empty(n_turns), turn_n=np.empty(n_turns, np.int64), turn_cum=np.empty(n_turns),
             traj_cum=np.empty(n_traj), stop_turn=np.empty(n_traj, np.int32),
-            stop_row=np.empty(n_traj, np.int64), row_cum=np.empty(logp_t.shape[0]))
+            stop_row=np.empty(n_traj, np.int64), traj_loss=np.empty(n_traj),
+            traj_loss_tokens=np.empty(n_traj, np.int64), row_cum=np.empty(logp_t.shape[0]),
+            profile=np.zeros(30))
         rc = self.lib.oracle_scan_batch(
-            _ptr(logp_t), _ptr(d), _ptr(tro), _ptr(uro), _ptr(tto), n_traj, mode, _ptr(lam_a),
-            _ptr(cin), _ptr(out["turn_sum_t"]), _ptr(out["turn_sum_d"]), _ptr(out["turn_mean"]),
-            _ptr(out["turn_n"]), _ptr(out["turn_cum"]), _ptr(out["traj_cum"]),
-            _ptr(out["stop_turn"]), _ptr(out["stop_row"]), _ptr(out["row_cum"]))
+            _ptr(logp_t), _ptr(d), _ptr(ls), _ptr(tro), _ptr(uro), _ptr(tto), n_traj, mode, _ptr(lam_a),
+            _ptr(cin), _ptr(out["turn_sum_t"]), _ptr(out["turn_sum_d"]), _ptr(out["turn_sum_l"]),
+            _ptr(out["turn_mean"]), _ptr(out["turn_n"]), _ptr(out["turn_cum"]), _ptr(out["traj_cum"]),
+            _ptr(out["stop_turn"]), _ptr(out["stop_row"]), _ptr(out["traj_loss"]),
+            _ptr(out["traj_loss_tokens"]), _ptr(out["row_cum"]), _ptr(out["profile"]))
         if rc != OK:
             raise ValueError(f"oracle_scan_batch returned {rc}")
+        out["profile"] = out["profile"].reshape(10, 3)
         return out
 
     # ---- Algorithm 1 inner loop: one decode step ---------------------------
@@ -151,13 +157,13 @@ class OracleLib:
         lam_a = np.ascontiguousarray(np.broadcast_to(np.asarray(lam, np.float64), (B,)))
         out = dict(logp_s=np.empty(B), logp_t=np.empty(B), d=np.empty(B),
                    stopped_now=np.empty(B, np.uint8), turn_sum_t=np.empty(B),
-                   turn_sum_d=np.empty(B), turn_mean=np.empty(B), turn_n=np.empty(B, np.int32),
-                   turn_cum=np.empty(B))
+                   turn_sum_d=np.empty(B), turn_sum_l=np.empty(B), turn_mean=np.empty(B),
+                   turn_n=np.empty(B, np.int32), turn_cum=np.empty(B))
         rc = self.lib.oracle_step_update(
             _ptr(ps), _ptr(pt), _ptr(te), B, mode, _ptr(lam_a), ctypes.cast(state, ctypes.c_void_p),
             _ptr(out["logp_s"]), _ptr(out["logp_t"]), _ptr(out["d"]), _ptr(out["stopped_now"]),
-            _ptr(out["turn_sum_t"]), _ptr(out["turn_sum_d"]), _ptr(out["turn_mean"]),
-            _ptr(out["turn_n"]), _ptr(out["turn_cum"]))
+            _ptr(out["turn_sum_t"]), _ptr(out["turn_sum_d"]), _ptr(out["turn_sum_l"]),
+            _ptr(out["turn_mean"]), _ptr(out["turn_n"]), _ptr(out["turn_cum"]))
         if rc != OK:
             raise ValueError(f"oracle_step_update returned {rc}")
         return out
@@ -184,7 +190,8 @@ class OracleLib:
 class Rollouts(ctypes.Structure):
     """Mirror of the oracle's own per-rollout step state."""
     _fields_ = [("cum", ctypes.c_double), ("turn_sum_t", ctypes.c_double),
-                ("turn_sum_d", ctypes.c_double), ("rows_seen", ctypes.c_int64),
+                ("turn_sum_d", ctypes.c_double), ("turn_sum_l", ctypes.c_double),
+                ("loss", ctypes.c_double), ("rows_seen", ctypes.c_int64),
                 ("stop_row", ctypes.c_int64), ("stop_turn", ctypes.c_int32),
                 ("turn_tokens", ctypes.c_int32), ("turn_idx", ctypes.c_int32),
                 ("stopped", ctypes.c_int32)]

@@ -19,6 +19,12 @@
  *                         offset (Sec. 4.1, "Synergy with the prefix buffer":
  *                         the sum runs over newly generated turns only); the
  *                         token-level variant used for math (Sec. 5.5).
+ *                         Also the token-level OPD loss of Eq. 2 on the
+ *                         retained tokens (Algorithm 1: the loss covers the
+ *                         tokens kept, including the triggering turn), per
+ *                         turn and per trajectory, and the within-turn
+ *                         relative-position decile profile of d and log pi_T
+ *                         (Observation 1, Sec. 3.2).
  *   oracle_step_update    the same rules applied online, one generated token
  *                         per rollout per call (Algorithm 1, inner turn loop).
  *   oracle_select_restart quality gate l_k > alpha (Sec. 4.2, step 1), the
@@ -199,16 +205,31 @@ int oracle_row_logprobs(const void* S, const void* T, int dtype, int64_t ld, int
  * Turns after the stop are still summarised (they are reported, not scored
  * differently); only the first crossing is recorded.
  *
- * Outputs (each may be NULL): per turn sum_t, sum_d, mean (fp64), n, cum after
- * the turn; per trajectory final cum, stop_turn (trajectory-local, -1 none),
- * stop_row (trajectory-local token position, -1 none); per row row_cum =
- * running token sum (TOKEN_SUM) or the turn-end running sum at turn-end rows
- * and NaN elsewhere (TURN_MEAN). */
-int oracle_scan_batch(const double* logp_t, const double* d, const int64_t* traj_row_off,
-                      const int64_t* turn_row_off, const int32_t* traj_turn_off, int32_t n_traj,
-                      int mode, const double* lambda, const double* cum_in, double* turn_sum_t,
-                      double* turn_sum_d, double* turn_mean, int64_t* turn_n, double* turn_cum,
-                      double* traj_cum, int32_t* stop_turn, int64_t* stop_row, double* row_cum) {
+ * OPD loss (Eq. 2, r_t = logp_T - logp_S held constant): the per-token term
+ * -logp_S(t) * r_t = logp_S(t) * d(t).  turn_sum_l is its sum over each turn;
+ * traj_loss / traj_loss_tokens sum it over the retained tokens: every token
+ * of the turns up to and including the stopping turn (TURN_MEAN), every token
+ * up to and including the stopping token (TOKEN_SUM), all tokens if the rule
+ * never fires (Algorithm 1, loss on the retained tokens).
+ *
+ * Within-turn profile (Observation 1): token i (0-based) of a turn of n_k
+ * tokens falls in decile floor(10 i / n_k); profile[3j+0] += d, profile[3j+1]
+ * += logp_T, profile[3j+2] += 1 for its decile j.  The profile is added to
+ * (not cleared).
+ *
+ * Outputs (each may be NULL): per turn sum_t, sum_d, sum_l, mean (fp64), n,
+ * cum after the turn; per trajectory final cum, stop_turn (trajectory-local,
+ * -1 none), stop_row (trajectory-local token position, -1 none), retained
+ * loss and token count; per row row_cum = running token sum (TOKEN_SUM) or
+ * the turn-end running sum at turn-end rows and NaN elsewhere (TURN_MEAN);
+ * profile [30].  logp_s may be NULL when the loss outputs are not wanted. */
+int oracle_scan_batch(const double* logp_t, const double* d, const double* logp_s,
+                      const int64_t* traj_row_off, const int64_t* turn_row_off,
+                      const int32_t* traj_turn_off, int32_t n_traj, int mode, const double* lambda,
+                      const double* cum_in, double* turn_sum_t, double* turn_sum_d,
+                      double* turn_sum_l, double* turn_mean, int64_t* turn_n, double* turn_cum,
+                      double* traj_cum, int32_t* stop_turn, int64_t* stop_row, double* traj_loss,
+                      int64_t* traj_loss_tokens, double* row_cum, double* profile) {
   if (!logp_t || !traj_row_off || !turn_row_off || !traj_turn_off || !lambda || n_traj < 0)
     return ORACLE_ERR_ARG;
   if (mode != ORACLE_MODE_TURN_MEAN && mode != ORACLE_MODE_TOKEN_SUM) return ORACLE_ERR_ARG;
@@ -221,25 +242,48 @@ int oracle_scan_batch(const double* logp_t, const double* d, const int64_t* traj
     double cum = cum_in ? cum_in[i] : 0.0;
     int32_t st_turn = -1;
     int64_t st_row = -1;
+    double loss = 0.0;
+    int64_t loss_n = 0;
     for (int32_t k = k0; k < k1; ++k) {
       int64_t a = turn_row_off[k], b = turn_row_off[k + 1];
       if (b <= a) return ORACLE_ERR_EMPTY_TURN; /* Eq. 4 needs n_k >= 1 */
-      double s_t = 0.0, s_d = 0.0;
+      int64_t n = b - a;
+      /* a turn (TURN_MEAN) or a token (TOKEN_SUM) is retained when the rule
+       * has not fired before it */
+      int turn_retained = (st_turn < 0);
+      double s_t = 0.0, s_d = 0.0, s_l = 0.0;
       for (int64_t r = a; r < b; ++r) {
-        s_t += logp_t[r - base];
-        if (d) s_d += d[r - base];
+        double lt = logp_t[r - base];
+        double dd = d ? d[r - base] : 0.0;
+        double term = logp_s ? logp_s[r - base] * dd : 0.0; /* -logp_S * r_t (Eq. 2) */
+        s_t += lt;
+        s_d += dd;
+        s_l += term;
+        if (profile) {
+          int64_t j = (10 * (r - a)) / n;
+          profile[3 * j + 0] += dd;
+          profile[3 * j + 1] += lt;
+          profile[3 * j + 2] += 1.0;
+        }
         if (mode == ORACLE_MODE_TOKEN_SUM) {
-          cum += logp_t[r - base];
+          if (st_row < 0) {
+            loss += term;
+            loss_n += 1;
+          }
+          cum += lt;
           if (row_cum) row_cum[r - base] = cum;
           if (st_row < 0 && cum < lambda[i]) {
             st_row = r - traj_row_off[i];
             st_turn = k - k0;
           }
-        } else if (row_cum) {
-          row_cum[r - base] = NAN;
+        } else {
+          if (turn_retained) {
+            loss += term;
+            loss_n += 1;
+          }
+          if (row_cum) row_cum[r - base] = NAN;
         }
       }
-      int64_t n = b - a;
       double mean = s_t / (double)n; /* Eq. 4 */
       if (mode == ORACLE_MODE_TURN_MEAN) {
         cum += mean; /* Eq. 5 left-hand side, over new turns only */
@@ -251,6 +295,7 @@ int oracle_scan_batch(const double* logp_t, const double* d, const int64_t* traj
       }
       if (turn_sum_t) turn_sum_t[k] = s_t;
       if (turn_sum_d) turn_sum_d[k] = s_d;
+      if (turn_sum_l) turn_sum_l[k] = s_l;
       if (turn_mean) turn_mean[k] = mean;
       if (turn_n) turn_n[k] = n;
       if (turn_cum) turn_cum[k] = cum;
@@ -258,6 +303,8 @@ int oracle_scan_batch(const double* logp_t, const double* d, const int64_t* traj
     if (traj_cum) traj_cum[i] = cum;
     if (stop_turn) stop_turn[i] = st_turn;
     if (stop_row) stop_row[i] = st_row;
+    if (traj_loss) traj_loss[i] = loss;
+    if (traj_loss_tokens) traj_loss_tokens[i] = loss_n;
   }
   return ORACLE_OK;
 }
@@ -267,7 +314,9 @@ typedef struct {
   double cum;        /* running sum (Eq. 5 left-hand side, or token sum) */
   double turn_sum_t; /* open turn: sum of logp_T */
   double turn_sum_d; /* open turn: sum of d */
-  int64_t rows_seen; /* tokens scored so far */
+  double turn_sum_l; /* open turn: sum of the OPD-loss terms logp_S * d */
+  double loss;       /* OPD loss (Eq. 2) over the tokens scored, all retained */
+  int64_t rows_seen; /* tokens scored so far (= retained tokens) */
   int64_t stop_row;  /* token position of the first crossing, -1 none */
   int32_t stop_turn; /* turn of the first crossing, -1 none */
   int32_t turn_tokens;
@@ -282,12 +331,14 @@ typedef struct {
  * TOKEN_SUM tests the running sum at every token, and when turn_end[b] is set
  * the turn closes: l = sum_t / n (Eq. 4), TURN_MEAN adds l to the running sum
  * and tests it (Eq. 5).  A closed turn's stats are reported in the turn_*
- * outputs (turn_n = 0 when no turn closed at this step). */
+ * outputs (turn_n = 0 when no turn closed at this step).  Every scored token
+ * is retained (a stopped rollout scores nothing more), so its OPD-loss term
+ * logp_S * d (Eq. 2) is added to the rollout's loss. */
 int oracle_step_update(const double* logp_s, const double* logp_t, const uint8_t* turn_end,
                        int32_t B, int mode, const double* lambda, oracle_rollout* st,
                        double* out_logp_s, double* out_logp_t, double* out_d, uint8_t* stopped_now,
-                       double* turn_sum_t, double* turn_sum_d, double* turn_mean, int32_t* turn_n,
-                       double* turn_cum) {
+                       double* turn_sum_t, double* turn_sum_d, double* turn_sum_l, double* turn_mean,
+                       int32_t* turn_n, double* turn_cum) {
   if (!logp_s || !logp_t || !turn_end || !lambda || !st || B < 0) return ORACLE_ERR_ARG;
   for (int32_t b = 0; b < B; ++b) {
     oracle_rollout* s = &st[b];
@@ -295,6 +346,7 @@ int oracle_step_update(const double* logp_s, const double* logp_t, const uint8_t
     if (turn_n) turn_n[b] = 0;
     if (turn_sum_t) turn_sum_t[b] = 0.0;
     if (turn_sum_d) turn_sum_d[b] = 0.0;
+    if (turn_sum_l) turn_sum_l[b] = 0.0;
     if (turn_mean) turn_mean[b] = 0.0;
     if (turn_cum) turn_cum[b] = 0.0;
     if (s->stopped) {
@@ -309,6 +361,8 @@ int oracle_step_update(const double* logp_s, const double* logp_t, const uint8_t
     if (out_d) out_d[b] = dd;
     s->turn_sum_t += pt;
     s->turn_sum_d += dd;
+    s->turn_sum_l += ps * dd;
+    s->loss += ps * dd;
     s->turn_tokens += 1;
     int64_t pos = s->rows_seen;
     s->rows_seen += 1;
@@ -335,12 +389,14 @@ int oracle_step_update(const double* logp_s, const double* logp_t, const uint8_t
       if (turn_n) turn_n[b] = s->turn_tokens;
       if (turn_sum_t) turn_sum_t[b] = s->turn_sum_t;
       if (turn_sum_d) turn_sum_d[b] = s->turn_sum_d;
+      if (turn_sum_l) turn_sum_l[b] = s->turn_sum_l;
       if (turn_mean) turn_mean[b] = mean;
       if (turn_cum) turn_cum[b] = s->cum;
       s->turn_idx += 1;
       s->turn_tokens = 0;
       s->turn_sum_t = 0.0;
       s->turn_sum_d = 0.0;
+      s->turn_sum_l = 0.0;
     }
   }
   return ORACLE_OK;

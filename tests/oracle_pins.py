@@ -238,6 +238,69 @@ def check_stop_rule_golden(orc):
         assert int(o["stop_row"][0]) == c["stop_row"], (c["name"], o["stop_row"])
 
 
+def _loss_cases():
+    return json.loads((GOLD / "opd_loss_cases.json").read_text())
+
+
+def check_opd_loss_golden(orc):
+    """Retained-token OPD loss (Eq. 2, Algorithm 1) on hand-worked cases."""
+    for c in _loss_cases()["cases"]:
+        lay = layout_from_turn_lengths([[len(t) for t in c["turns"]]])
+        rows = np.array([r for t in c["turns"] for r in t], np.float64)
+        ls, lt = rows[:, 0], rows[:, 1]
+        mode = oracle.TURN_MEAN if c["mode"] == "turn_mean" else oracle.TOKEN_SUM
+        o = orc.scan_batch(lt, ls - lt, lay.traj_row_off, lay.turn_row_off, lay.traj_turn_off, mode, c["lambda"],
+                           logp_s=ls)
+        assert list(o["turn_sum_l"]) == c["turn_sum_l"], (c["name"], o["turn_sum_l"])
+        assert o["traj_loss"][0] == c["loss"], (c["name"], o["traj_loss"])
+        assert int(o["traj_loss_tokens"][0]) == c["loss_tokens"], c["name"]
+        assert int(o["stop_turn"][0]) == c["stop_turn"], c["name"]
+
+
+def check_turn_profile_golden(orc):
+    """Within-turn decile profile (Observation 1) on a hand-worked case."""
+    pc = _loss_cases()["profile_case"]
+    lay = layout_from_turn_lengths([pc["turn_lengths"]])
+    d = np.concatenate([np.arange(20.0), [100.0, 200.0, 300.0]])
+    lt = np.concatenate([np.full(20, -1.0), np.full(3, -4.0)])
+    o = orc.scan_batch(lt, d, lay.traj_row_off, lay.turn_row_off, lay.traj_turn_off, oracle.TURN_MEAN, -1e300)
+    assert np.array_equal(o["profile"], np.array(pc["profile"])), o["profile"]
+
+
+def check_loss_invariants(orc):
+    """Loss over all tokens when the rule never fires; in turn mode the
+    retained loss is the sum of turn sums up to the stopping turn; in token
+    mode the sum of terms up to the stopping token; profile counts sum to the
+    rows and its d column to the sum of d."""
+    for seed in range(4):
+        lay, lp, d = _random_scan_data(400 + seed)
+        ls = lp + d
+        terms = ls * d
+        for mode, lam in ((oracle.TURN_MEAN, -4.0), (oracle.TOKEN_SUM, -30.0)):
+            never = orc.scan_batch(lp, d, lay.traj_row_off, lay.turn_row_off, lay.traj_turn_off, mode, -1e300,
+                                   logp_s=ls)
+            o = orc.scan_batch(lp, d, lay.traj_row_off, lay.turn_row_off, lay.traj_turn_off, mode, lam, logp_s=ls)
+            assert int(o["profile"][:, 2].sum()) == lay.rows
+            assert abs(o["profile"][:, 0].sum() - math.fsum(d)) <= 1e-9 * math.fsum(np.abs(d))
+            for i in range(lay.n_traj):
+                r0, r1 = lay.traj_row_off[i], lay.traj_row_off[i + 1]
+                k0, k1 = lay.traj_turn_off[i], lay.traj_turn_off[i + 1]
+                assert abs(never["traj_loss"][i] - math.fsum(terms[r0:r1])) <= 1e-9 * (1 + math.fsum(np.abs(terms[r0:r1])))
+                assert never["traj_loss_tokens"][i] == r1 - r0
+                if o["stop_row"][i] < 0:
+                    assert o["traj_loss_tokens"][i] == r1 - r0
+                    continue
+                if mode == oracle.TURN_MEAN:
+                    kk = k0 + int(o["stop_turn"][i])
+                    want = math.fsum(o["turn_sum_l"][k0:kk + 1])
+                    n = int(lay.turn_row_off[kk + 1] - r0)
+                else:
+                    n = int(o["stop_row"][i]) + 1
+                    want = math.fsum(terms[r0:r0 + n])
+                assert o["traj_loss_tokens"][i] == n
+                assert abs(o["traj_loss"][i] - want) <= 1e-9 * (1 + abs(want))
+
+
 def check_prefix_buffer_offset(orc):
     """Scanning only the new turns after K0 reused turns (Sec. 4.1) differs
     from scanning the whole record, as the golden derivation states."""
@@ -362,8 +425,13 @@ def check_step_matches_batch(orc):
         lay, lp, d = _random_scan_data(300 + seed, n_traj=6)
         for mode, lam in ((oracle.TURN_MEAN, -4.0), (oracle.TOKEN_SUM, -30.0)):
             ob = orc.scan_batch(lp, d, lay.traj_row_off, lay.turn_row_off, lay.traj_turn_off, mode, lam)
+            obl = orc.scan_batch(lp, d, lay.traj_row_off, lay.turn_row_off, lay.traj_turn_off, mode, lam,
+                                 logp_s=lp + d)
             st, outs, _ = _run_steps(orc, lay, lp, d, mode, lam)
             for b in range(lay.n_traj):
+                # every token a rollout scores is retained: its loss is the batch retained loss
+                assert abs(st[b].loss - obl["traj_loss"][b]) <= 1e-9 * (1 + abs(obl["traj_loss"][b])), (seed, mode, b)
+                assert st[b].rows_seen == obl["traj_loss_tokens"][b] or st[b].stop_row < 0
                 assert st[b].stop_turn == ob["stop_turn"][b], (seed, mode, b)
                 assert st[b].stop_row == ob["stop_row"][b], (seed, mode, b)
                 if st[b].stop_row >= 0:
@@ -434,6 +502,7 @@ ALL_CHECKS = [
     check_teacher_only, check_bf16_decode, check_special_values, check_strided_rows,
     check_stop_rule_golden, check_prefix_buffer_offset, check_scan_invariants,
     check_traj_independence, check_per_trajectory_lambda, check_empty_turn_rejected,
+    check_opd_loss_golden, check_turn_profile_golden, check_loss_invariants,
     check_step_matches_batch, check_step_golden,
     check_select_golden, check_select_bruteforce,
 ]

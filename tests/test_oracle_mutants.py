@@ -38,6 +38,13 @@ MUTANTS = [
     ("select_kmax_all_turns", "while (K < nt && (m == NULL || m[K] != 0) && (l[K] > alpha)) ++K;",
      "for (int32_t q = 0; q < nt; ++q) if ((m == NULL || m[q] != 0) && (l[q] > alpha)) ++K;"),
     ("select_argmax", "if (l[k] < l[best]) best = k;", "if (l[k] > l[best]) best = k;"),
+    ("loss_sign", "double term = logp_s ? logp_s[r - base] * dd : 0.0;", "double term = logp_s ? -logp_s[r - base] * dd : 0.0;"),
+    ("loss_uses_teacher", "double term = logp_s ? logp_s[r - base] * dd : 0.0;", "double term = logp_s ? lt * dd : 0.0;"),
+    ("loss_all_turns_retained", "int turn_retained = (st_turn < 0);", "int turn_retained = 1;"),
+    ("loss_drops_trigger_token", "if (st_row < 0) {\n            loss += term;",
+     "if (st_row < 0 && cum + lt >= lambda[i]) {\n            loss += term;"),
+    ("profile_wrong_decile", "int64_t j = (10 * (r - a)) / n;", "int64_t j = (10 * (r - a)) / (n + 1);"),
+    ("step_loss_teacher", "s->loss += ps * dd;", "s->loss += pt * dd;"),
 ]
 
 
