@@ -17,7 +17,12 @@
  *                                  first token whose running teacher log-prob
  *                                  falls below lambda (Sec. 5.5);
  *   k*, K_max                      the weakest correct turn of Eq. 6 behind
- *                                  the quality gate of Sec. 4.2.
+ *                                  the quality gate of Sec. 4.2;
+ *   OPD loss                       the token-level loss of Eq. 2 on the
+ *                                  retained tokens (Algorithm 1: the tokens
+ *                                  kept, including the triggering turn);
+ *   within-turn profile            d and log pi_T by relative position within
+ *                                  a turn, in deciles (Observation 1).
  *
  * Conventions shared by every entry point
  * ---------------------------------------
@@ -56,7 +61,7 @@
 extern "C" {
 #endif
 
-#define STRIDE_ABI_VERSION 1
+#define STRIDE_ABI_VERSION 2
 
 #if defined(__GNUC__)
 #define STRIDE_API __attribute__((visibility("default")))
@@ -87,17 +92,24 @@ typedef enum stride_status {
 #define STRIDE_STOP_TURN_MEAN 0 /* Eq. 5: running sum of per-turn means l_k, tested at turn ends */
 #define STRIDE_STOP_TOKEN_SUM 1 /* Sec. 5.5: running sum of token log-probs, tested at every token */
 
-/* ---- per-trajectory / per-rollout carried state (56 bytes) ---------------
+/* ---- per-trajectory / per-rollout carried state (80 bytes) ---------------
  * Initialise with stride_state_init.  It is both the carry between calls
  * (chunked batch scoring, decode steps) and the per-trajectory result.
  * A trajectory's running sum starts from `cum` at its first row (0 after
  * init), which is how the prefix-buffer offset is expressed: pass only the
- * newly generated turns of a restarted rollout (Sec. 4.1; Algorithm 1). */
+ * newly generated turns of a restarted rollout (Sec. 4.1; Algorithm 1).
+ * `loss` accumulates the OPD-loss terms logp_S * d (= -log pi_S * r_t, Eq. 2)
+ * of the retained tokens: in turn mode every token of the turns up to and
+ * including the triggering turn, in token mode every token up to and
+ * including the triggering token, all tokens while the rule has not fired. */
 typedef struct stride_scan_state {
   double cum;          /* running sum through the last scored token (Eq. 5 LHS or token sum) */
   double turn_sum_t;   /* open turn: sum of log pi_T so far */
   double turn_sum_d;   /* open turn: sum of d so far */
+  double turn_sum_l;   /* open turn: sum of logp_S * d so far */
+  double loss;         /* OPD loss (Eq. 2) over the retained tokens scored so far */
   int64_t rows_seen;   /* tokens of this trajectory scored so far */
+  int64_t loss_tokens; /* retained tokens scored so far */
   int64_t stop_row;    /* token position (trajectory-local) of the first crossing; -1 = none */
   int32_t stop_turn;   /* turn (trajectory-local, 0-based) of the first crossing; -1 = none */
   int32_t turn_tokens; /* tokens in the open turn */
@@ -105,14 +117,22 @@ typedef struct stride_scan_state {
   int32_t stopped;     /* non-zero once the stop rule has fired */
 } stride_scan_state;
 
-/* ---- per-turn statistics (32 bytes) --------------------------------------- */
+/* ---- per-turn statistics (40 bytes) --------------------------------------- */
 typedef struct stride_turn_stats {
   double sum_t;  /* sum of log pi_T over the turn's tokens */
   double sum_d;  /* sum of d over the turn's tokens (turn mean KL = sum_d / n, Sec. 3.2) */
+  double sum_l;  /* sum of logp_S * d over the turn's tokens (the turn's OPD loss, Eq. 2) */
   double cum;    /* running sum after this turn (Eq. 5 LHS; token sum at the turn's end in TOKEN_SUM) */
   float mean_t;  /* l_k = sum_t / n (Eq. 4), rounded to fp32 */
   int32_t n;     /* tokens in the turn (n_k) */
 } stride_turn_stats;
+
+/* ---- within-turn position profile ------------------------------------------
+ * double [STRIDE_PROFILE_BINS][3]: for each decile j of relative position in
+ * a turn (token i of a turn of n tokens is in decile floor(10 i / n)), the sum
+ * of d, the sum of log pi_T and the token count (Observation 1).  The
+ * scoring call ADDS to it; zero it before the first call. */
+#define STRIDE_PROFILE_BINS 10
 
 /* ---- optional per-row outputs (host struct of device pointers) ------------
  * Each pointer is nullable; a non-NULL pointer receives one float per row. */
@@ -161,6 +181,7 @@ STRIDE_API size_t stride_score_batch_workspace_size(int64_t window_rows);
  * out: host struct of optional per-row outputs indexed by (row - row_begin); NULL for none.
  * turn_stats: device [n_turns] or NULL; turn k is written by the call that
  * scores its last row.
+ * profile: device double [STRIDE_PROFILE_BINS * 3] or NULL; added to.
  * dev_status: device int32 or NULL.
  * workspace: device, >= stride_score_batch_workspace_size(row_end-row_begin)
  * bytes, 256-byte aligned; it is cleared by the call, holds nothing between
@@ -172,8 +193,8 @@ STRIDE_API int stride_score_batch(const void* S, const void* T, int32_t dtype, i
                        int32_t n_turns, int64_t row_begin, int64_t row_end, int32_t stop_mode,
                        const float* lambda, float lambda_all, stride_scan_state* state,
                        const stride_row_outputs* out, stride_turn_stats* turn_stats,
-                       int32_t* dev_status, void* workspace, size_t workspace_bytes,
-                       void* stream);
+                       double* profile, int32_t* dev_status, void* workspace,
+                       size_t workspace_bytes, void* stream);
 
 /* One decode step over B rollouts (Algorithm 1, inner turn loop, one
  * generated token per rollout).
@@ -187,6 +208,7 @@ STRIDE_API int stride_score_batch(const void* S, const void* T, int32_t dtype, i
  *   TOKEN_SUM: cum += log pi_T; stop if cum < lambda;
  *   TURN_MEAN: at a turn end, l = turn_sum_t / turn_tokens (Eq. 4),
  *              cum += l, stop if cum < lambda (Eq. 5).
+ * Every scored token is retained, so its logp_S * d is added to state.loss.
  * stopped_now: uint8 [B] or NULL, 1 where the rule fired at this step.
  * turn_out: device [B] or NULL: the stats of the turn closed at this step
  * (n = 0 where none closed).  lambda / lambda_all as for stride_score_batch.
@@ -245,8 +267,8 @@ STRIDE_API int stride_score_batch_noalloc(const void* S, const void* T, int32_t 
                                           int32_t n_turns, int64_t row_begin, int64_t row_end,
                                           int32_t stop_mode, const float* lambda, float lambda_all,
                                           stride_scan_state* state, const stride_row_outputs* out,
-                                          stride_turn_stats* turn_stats, int32_t* dev_status,
-                                          void* stream);
+                                          stride_turn_stats* turn_stats, double* profile,
+                                          int32_t* dev_status, void* stream);
 
 /* Human-readable name of a stride_status code (static string). */
 STRIDE_API const char* stride_status_string(int code);

@@ -9,7 +9,7 @@ CPU fallback, and importing this package fails if the library is missing
 and cannot be built.
 
 Per-trajectory state and per-turn statistics are opaque byte tensors
-(``[n, 56]`` and ``[n, 32]`` uint8) laid out as ``stride_scan_state`` and
+(``[n, 80]`` and ``[n, 40]`` uint8) laid out as ``stride_scan_state`` and
 ``stride_turn_stats``; :func:`state_to_numpy` / :func:`turn_stats_to_numpy`
 view copies of them as numpy structured arrays.
 """
@@ -28,7 +28,8 @@ __all__ = [
     "new_turn_stats", "state_to_numpy", "turn_stats_to_numpy", "stride_state_init",
     "stride_score_batch_workspace_size", "stride_score_batch", "stride_score_step",
     "stride_select_restart", "stride_status_string", "stride_abi_version", "ROW_OUTPUT_KEYS",
-    "stride_score_batch_noalloc", "NOALLOC_MAX_ROWS", "ERR_TOO_LARGE",
+    "stride_score_batch_noalloc", "NOALLOC_MAX_ROWS", "ERR_TOO_LARGE", "PROFILE_BINS", "new_profile",
+    "stride_selftest_bounded_wait",
 ]
 
 DTYPE_BF16, DTYPE_F32 = 0, 1
@@ -39,11 +40,13 @@ NOALLOC_MAX_ROWS = 65536  # STRIDE_NOALLOC_MAX_ROWS
 ERR_TOO_LARGE = 6
 
 STATE_DTYPE = np.dtype([("cum", "<f8"), ("turn_sum_t", "<f8"), ("turn_sum_d", "<f8"),
-                        ("rows_seen", "<i8"), ("stop_row", "<i8"), ("stop_turn", "<i4"),
+                        ("turn_sum_l", "<f8"), ("loss", "<f8"), ("rows_seen", "<i8"),
+                        ("loss_tokens", "<i8"), ("stop_row", "<i8"), ("stop_turn", "<i4"),
                         ("turn_tokens", "<i4"), ("turn_idx", "<i4"), ("stopped", "<i4")])
-TURN_STATS_DTYPE = np.dtype([("sum_t", "<f8"), ("sum_d", "<f8"), ("cum", "<f8"),
+TURN_STATS_DTYPE = np.dtype([("sum_t", "<f8"), ("sum_d", "<f8"), ("sum_l", "<f8"), ("cum", "<f8"),
                              ("mean_t", "<f4"), ("n", "<i4")])
-assert STATE_DTYPE.itemsize == 56 and TURN_STATS_DTYPE.itemsize == 32
+PROFILE_BINS = 10
+assert STATE_DTYPE.itemsize == 80 and TURN_STATS_DTYPE.itemsize == 40
 
 
 class StrideError(RuntimeError):
@@ -74,13 +77,13 @@ def lib() -> ctypes.CDLL:
         L.stride_score_batch_workspace_size.argtypes = [i64]
         L.stride_score_batch_workspace_size.restype = sz
         L.stride_score_batch.argtypes = [P, P, i32, i64, i64, P, P, P, P, i32, i32, i64, i64, i32, P, f32,
-                                         P, P, P, P, P, sz, P]
+                                         P, P, P, P, P, P, sz, P]
         L.stride_score_step.argtypes = [P, P, i32, i64, i64, P, P, i32, i32, P, f32, P, P, P, P, P, P]
         L.stride_select_restart.argtypes = [P, P, P, f32, i32, i32, P, P, P]
         L.stride_selftest_bounded_wait.argtypes = [i32, ctypes.c_uint64, P, P, sz, P]
         L.stride_selftest_bounded_wait.restype = ctypes.c_int
         L.stride_score_batch_noalloc.argtypes = [P, P, i32, i64, i64, P, P, P, P, i32, i32, i64, i64, i32,
-                                                 P, f32, P, P, P, P, P]
+                                                 P, f32, P, P, P, P, P, P]
         L.stride_status_string.argtypes = [ctypes.c_int]
         L.stride_status_string.restype = ctypes.c_char_p
         L.stride_abi_version.restype = ctypes.c_int
@@ -190,6 +193,12 @@ def new_turn_stats(n: int, device="cuda"):
     return torch.zeros((max(n, 1), TURN_STATS_DTYPE.itemsize), dtype=torch.uint8, device=device)
 
 
+def new_profile(device="cuda"):
+    """A zeroed within-turn position profile: float64 [PROFILE_BINS, 3]."""
+    torch = _torch()
+    return torch.zeros((PROFILE_BINS, 3), dtype=torch.float64, device=device)
+
+
 def state_to_numpy(st) -> np.ndarray:
     return st.detach().cpu().numpy().reshape(-1).view(STATE_DTYPE)
 
@@ -214,7 +223,7 @@ def stride_score_batch_workspace_size(window_rows: int) -> int:
 def stride_score_batch(S, T, tokens, traj_row_off, turn_row_off, traj_turn_off, row_begin: int,
                        row_end: int, stop_mode: int, lam, state, out: dict | None = None,
                        turn_stats=None, dev_status=None, workspace=None, V: int | None = None,
-                       stream=None) -> None:
+                       stream=None, profile=None) -> None:
     """Score global rows [row_begin, row_end) of a ragged trajectory layout.
 
     S, T: [row_end-row_begin, ld] bf16/fp32 logits of those rows; tokens int32;
@@ -223,7 +232,8 @@ def stride_score_batch(S, T, tokens, traj_row_off, turn_row_off, traj_turn_off, 
     of float32 [rows] tensors keyed by ROW_OUTPUT_KEYS; turn_stats from
     :func:`new_turn_stats`; dev_status an int32 [1] tensor; workspace a uint8
     tensor of at least stride_score_batch_workspace_size(rows) bytes (256-byte
-    aligned; torch's allocator returns such blocks)."""
+    aligned; torch's allocator returns such blocks); profile a float64
+    [10, 3] tensor from :func:`new_profile`, added to."""
     torch = _torch()
     dt, ld = _logits(S, T)
     rows = int(row_end) - int(row_begin)
@@ -239,6 +249,7 @@ def stride_score_batch(S, T, tokens, traj_row_off, turn_row_off, traj_turn_off, 
         int(row_end), int(stop_mode), lam_p, lam_all,
         _dev(state, "state", torch.uint8, n_traj * STATE_DTYPE.itemsize), _row_outputs(out, rows),
         _dev(turn_stats, "turn_stats", torch.uint8, n_turns * TURN_STATS_DTYPE.itemsize, optional=True),
+        _dev(profile, "profile", torch.float64, 3 * PROFILE_BINS, optional=True),
         _dev(dev_status, "dev_status", torch.int32, 1, optional=True), ws_p,
         0 if workspace is None else workspace.numel(), _stream(stream))
     _check("stride_score_batch", rc)
@@ -291,7 +302,8 @@ def stride_selftest_bounded_wait(which: int, timeout_ns: int, dev_status, worksp
 
 def stride_score_batch_noalloc(S, T, tokens, traj_row_off, turn_row_off, traj_turn_off, row_begin: int,
                                row_end: int, stop_mode: int, lam, state, out: dict | None = None,
-                               turn_stats=None, dev_status=None, V: int | None = None, stream=None) -> None:
+                               turn_stats=None, dev_status=None, V: int | None = None, stream=None,
+                               profile=None) -> None:
     """stride_score_batch without a workspace argument, for callers that
     cannot allocate device memory: the library's built-in scratch (at most
     NOALLOC_MAX_ROWS rows per call) is used instead.  Calls that overlap on
@@ -310,5 +322,6 @@ def stride_score_batch_noalloc(S, T, tokens, traj_row_off, turn_row_off, traj_tu
         int(row_end), int(stop_mode), lam_p, lam_all,
         _dev(state, "state", torch.uint8, n_traj * STATE_DTYPE.itemsize), _row_outputs(out, max(rows, 0)),
         _dev(turn_stats, "turn_stats", torch.uint8, n_turns * TURN_STATS_DTYPE.itemsize, optional=True),
+        _dev(profile, "profile", torch.float64, 3 * PROFILE_BINS, optional=True),
         _dev(dev_status, "dev_status", torch.int32, 1, optional=True), _stream(stream))
     _check("stride_score_batch_noalloc", rc)

@@ -94,8 +94,8 @@ int stride_score_batch(const void* S, const void* T, int32_t dtype, int64_t ld, 
                        int32_t n_turns, int64_t row_begin, int64_t row_end, int32_t stop_mode,
                        const float* lambda, float lambda_all, stride_scan_state* state,
                        const stride_row_outputs* out, stride_turn_stats* turn_stats,
-                       int32_t* dev_status, void* workspace, size_t workspace_bytes,
-                       void* stream) {
+                       double* profile, int32_t* dev_status, void* workspace,
+                       size_t workspace_bytes, void* stream) {
   const int lc = check_logits(S, T, dtype, ld, V);
   if (lc != STRIDE_OK) return lc;
   if (row_begin < 0 || row_end < row_begin || row_end - row_begin > INT32_MAX)
@@ -136,6 +136,7 @@ int stride_score_batch(const void* S, const void* T, int32_t dtype, int64_t ld, 
   p.state = state;
   p.out = row_outputs(out);
   p.turn_stats = turn_stats;
+  p.profile = profile;
   p.dev_status = dev_status;
   p.ticket = reinterpret_cast<uint32_t*>(ws + L.ticket_off);
   p.flags = reinterpret_cast<uint32_t*>(ws + L.flags_off);

@@ -42,17 +42,19 @@ struct ScanElem {
   double c;   // running stop-sum terms
   double st;  // sum of log pi_T within the open turn
   double sd;  // sum of d within the open turn
+  double sl;  // sum of the OPD-loss terms logp_S * d within the open turn
   int fturn;  // the range contains a turn's first row
 };
 
 // a (earlier rows) (+) b (later rows).  c never resets inside a lookback
-// (trajectory starts publish inclusive prefixes); st and sd restart at a
+// (trajectory starts publish inclusive prefixes); st, sd and sl restart at a
 // turn's first row.
 __device__ __forceinline__ ScanElem combine(const ScanElem& a, const ScanElem& b) {
   ScanElem r;
   r.c = a.c + b.c;
   r.st = b.fturn ? b.st : a.st + b.st;
   r.sd = b.fturn ? b.sd : a.sd + b.sd;
+  r.sl = b.fturn ? b.sl : a.sl + b.sl;
   r.fturn = a.fturn | b.fturn;
   return r;
 }
@@ -72,6 +74,7 @@ __device__ __forceinline__ void publish(ScanSlot* slot, uint32_t* flag, const Sc
   slot->c = e.c;
   slot->st = e.st;
   slot->sd = e.sd;
+  slot->sl = e.sl;
   st_release_u32(flag, status);
 }
 
@@ -153,7 +156,7 @@ __device__ __forceinline__ void validate_layout(const BatchParams& p, int64_t t)
 // Folds published predecessors of `tile` back to the nearest inclusive
 // prefix.  Warp-wide; every lane returns the same exclusive prefix.
 static __device__ ScanElem lookback(const BatchParams& p, int64_t tile, int lane, bool& timed_out) {
-  ScanElem excl = {0.0, 0.0, 0.0, 0};
+  ScanElem excl = {0.0, 0.0, 0.0, 0.0, 0};
   int64_t j = tile - 1;
   const uint64_t t0 = globaltimer_ns();
   while (true) {
@@ -174,7 +177,7 @@ static __device__ ScanElem lookback(const BatchParams& p, int64_t tile, int lane
     const bool is_incl = (f & kStMask) == kStIncl;
     const unsigned inc = __ballot_sync(0xffffffffu, is_incl);
     const int stop = inc ? __ffs(inc) - 1 : 31;
-    ScanElem v = {0.0, 0.0, 0.0, 0};
+    ScanElem v = {0.0, 0.0, 0.0, 0.0, 0};
     if (valid && lane <= stop && !(f & kFlagTimedOut)) {
       const ScanSlot* src = is_incl ? (p.incl + idx) : (p.agg + idx);
       const double2 a = __ldcg(reinterpret_cast<const double2*>(src));
@@ -182,6 +185,7 @@ static __device__ ScanElem lookback(const BatchParams& p, int64_t tile, int lane
       v.c = a.x;
       v.st = a.y;
       v.sd = b.x;
+      v.sl = b.y;
       v.fturn = (is_incl || (f & kFlagTurnStart)) ? 1 : 0;
     }
     if (f & kFlagTimedOut) timed_out = true;
@@ -193,6 +197,7 @@ static __device__ ScanElem lookback(const BatchParams& p, int64_t tile, int lane
       o.c = __shfl_down_sync(0xffffffffu, v.c, d);
       o.st = __shfl_down_sync(0xffffffffu, v.st, d);
       o.sd = __shfl_down_sync(0xffffffffu, v.sd, d);
+      o.sl = __shfl_down_sync(0xffffffffu, v.sl, d);
       o.fturn = __shfl_down_sync(0xffffffffu, v.fturn, d);
       if (lane + d < 32) v = combine(o, v);
     }
@@ -200,6 +205,7 @@ static __device__ ScanElem lookback(const BatchParams& p, int64_t tile, int lane
     win.c = __shfl_sync(0xffffffffu, v.c, 0);
     win.st = __shfl_sync(0xffffffffu, v.st, 0);
     win.sd = __shfl_sync(0xffffffffu, v.sd, 0);
+    win.sl = __shfl_sync(0xffffffffu, v.sl, 0);
     win.fturn = __shfl_sync(0xffffffffu, v.fturn, 0);
     excl = combine(win, excl);
     if (inc) break;
@@ -211,18 +217,23 @@ static __device__ ScanElem lookback(const BatchParams& p, int64_t tile, int lane
 
 
 // The part of a row's tail that waits on nobody: outputs, the row's scan
-// element, and its publication (an AGGREGATE, or, for a tile that starts a
-// trajectory or the window, the INCLUSIVE prefix seeded from the carried
-// state).  Lane 0 only.
+// element, the within-turn profile, and the element's publication (an
+// AGGREGATE, or, for a tile that starts a trajectory or the window, the
+// INCLUSIVE prefix seeded from the carried state).  Lane 0 only.  `prof`
+// (30 doubles, or NULL) receives the profile: with atomics when it is the
+// caller's global array, plainly when it is one writer's shared copy.
 struct RowCarry {
   ScanElem e;
-  ScanElem incl;
+  ScanElem incl;      // valid for seeded tiles
+  double c_before;    // running sum before this row (seeded tiles)
+  double st_before;   // open-turn sum of log pi_T before this row (seeded tiles)
   int seeded;
 };
 
 __device__ __forceinline__ RowCarry row_finalize(const BatchParams& p, int64_t tile, int64_t r,
                                                  const RowMeta& meta, int32_t y, float xs, float xt,
-                                                 float lse_s, float lse_t) {
+                                                 float lse_s, float lse_t, double* prof,
+                                                 bool prof_atomic) {
   RowCarry rc;
   const int64_t n_k = meta.turn_end - meta.turn_start;
   const float nan = __int_as_float(0x7fc00000);
@@ -247,9 +258,24 @@ __device__ __forceinline__ RowCarry row_finalize(const BatchParams& p, int64_t t
   e.c = (p.mode == STRIDE_STOP_TURN_MEAN) ? (double)lpt / (double)(n_k > 0 ? n_k : 1) : (double)lpt;
   e.st = (double)lpt;
   e.sd = (double)dd;
+  e.sl = (double)lps * (double)dd;  // -log pi_S * r_t (Eq. 2)
   e.fturn = (r == meta.turn_start) ? 1 : 0;
+  if (prof && !meta.bad) {
+    const int j = (int)((10 * (r - meta.turn_start)) / n_k);  // Observation 1 decile
+    if (prof_atomic) {
+      atomicAdd(prof + 3 * j + 0, e.sd);
+      atomicAdd(prof + 3 * j + 1, e.st);
+      atomicAdd(prof + 3 * j + 2, 1.0);
+    } else {
+      prof[3 * j + 0] += e.sd;
+      prof[3 * j + 1] += e.st;
+      prof[3 * j + 2] += 1.0;
+    }
+  }
   rc.e = e;
   rc.seeded = (tile == 0) || (r == meta.traj_start) || meta.bad;
+  rc.c_before = 0.0;
+  rc.st_before = 0.0;
   if (rc.seeded) {
     if (meta.bad) {
       rc.incl = e;  // NaN terms; nothing downstream of a bad row is meaningful
@@ -258,9 +284,13 @@ __device__ __forceinline__ RowCarry row_finalize(const BatchParams& p, int64_t t
       const double cum0 = __ldcg(&sp->cum);
       const double st0 = __ldcg(&sp->turn_sum_t);
       const double sd0 = __ldcg(&sp->turn_sum_d);
+      const double sl0 = __ldcg(&sp->turn_sum_l);
+      rc.c_before = cum0;
+      rc.st_before = e.fturn ? 0.0 : st0;
       rc.incl.c = cum0 + e.c;
       rc.incl.st = e.fturn ? e.st : st0 + e.st;
       rc.incl.sd = e.fturn ? e.sd : sd0 + e.sd;
+      rc.incl.sl = e.fturn ? e.sl : sl0 + e.sl;
       rc.incl.fturn = 1;
     }
     publish(p.incl + tile, p.flags + tile, rc.incl, kStIncl);
@@ -272,17 +302,28 @@ __device__ __forceinline__ RowCarry row_finalize(const BatchParams& p, int64_t t
 }
 
 // The part that waits: the lookback (warp-wide) for an unseeded tile, the
-// INCLUSIVE publication, then turn statistics, the stop test and the
-// carried state (lane 0).  rc is read in lane 0.
+// INCLUSIVE publication, then (lane 0) turn statistics, the stop test, the
+// row's OPD-loss term if the row is retained, and the carried state.
+//
+// Retention: a row is retained when the stop rule has not fired before it.
+// In token mode that is "the running sum before the row is >= lambda"; in
+// turn mode "the running sum through the previous turn is >= lambda", which
+// is the running sum before the row minus the row's turn's terms so far
+// (c_before - st_before / n_k).  The sums are monotone, so this selects
+// exactly the rows up to the first crossing (its turn, in turn mode).
+// rc is read in lane 0.
 __device__ __forceinline__ void row_resolve(const BatchParams& p, int64_t tile, int64_t r,
                                             const RowMeta& meta, RowCarry rc, int lane) {
   const int seeded = __shfl_sync(0xffffffffu, rc.seeded, 0);
   ScanElem incl = rc.incl;
+  double c_before = rc.c_before, st_before = rc.st_before;
   bool timed_out = false;
   if (!seeded) {
     const ScanElem excl = lookback(p, tile, lane, timed_out);
     if (lane == 0) {
       incl = combine(excl, rc.e);
+      c_before = excl.c;
+      st_before = rc.e.fturn ? 0.0 : excl.st;
       publish(p.incl + tile, p.flags + tile, incl, kStIncl);
     }
   }
@@ -291,12 +332,13 @@ __device__ __forceinline__ void row_resolve(const BatchParams& p, int64_t tile, 
   if (meta.bad) return;
   const int64_t n_k = meta.turn_end - meta.turn_start;
 
-  // ---- turn statistics, stop test, carried state (lane 0) ---------------
+  // ---- turn statistics, stop test, loss, carried state (lane 0) ---------
   const bool turn_last = (r == meta.turn_end - 1);
   if (turn_last && p.turn_stats) {
     stride_turn_stats ts;
     ts.sum_t = incl.st;
     ts.sum_d = incl.sd;
+    ts.sum_l = incl.sl;
     ts.cum = incl.c;
     ts.mean_t = (float)(incl.st / (double)n_k);
     ts.n = (int32_t)n_k;
@@ -311,10 +353,16 @@ __device__ __forceinline__ void row_resolve(const BatchParams& p, int64_t tile, 
     atomicMin(reinterpret_cast<unsigned int*>(&sp->stop_turn), (unsigned int)meta.local_turn);
     sp->stopped = 1;
   }
+  const double before = (p.mode == STRIDE_STOP_TOKEN_SUM) ? c_before : c_before - st_before / (double)n_k;
+  if (before >= (double)lam) {
+    atomicAdd(&sp->loss, rc.e.sl);
+    atomicAdd(reinterpret_cast<unsigned long long*>(&sp->loss_tokens), 1ull);
+  }
   if (r == meta.traj_end - 1 || r == p.row_end - 1) {
     sp->cum = incl.c;
     sp->turn_sum_t = turn_last ? 0.0 : incl.st;
     sp->turn_sum_d = turn_last ? 0.0 : incl.sd;
+    sp->turn_sum_l = turn_last ? 0.0 : incl.sl;
     sp->rows_seen = r - meta.traj_start + 1;
     sp->turn_idx = turn_last ? meta.local_turn + 1 : meta.local_turn;
     sp->turn_tokens = turn_last ? 0 : (int32_t)(r - meta.turn_start + 1);
@@ -327,7 +375,7 @@ __device__ __forceinline__ void finish_row(const BatchParams& p, int64_t tile, i
                                            const RowMeta& meta, int32_t y, float xs, float xt,
                                            float lse_s, float lse_t, int lane) {
   RowCarry rc;
-  if (lane == 0) rc = row_finalize(p, tile, r, meta, y, xs, xt, lse_s, lse_t);
+  if (lane == 0) rc = row_finalize(p, tile, r, meta, y, xs, xt, lse_s, lse_t, p.profile, true);
   row_resolve(p, tile, r, meta, rc, lane);
 }
 

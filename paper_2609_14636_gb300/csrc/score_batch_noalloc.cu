@@ -74,7 +74,7 @@ extern "C" STRIDE_API int stride_score_batch_noalloc(
     const int64_t* traj_row_off, const int64_t* turn_row_off, const int32_t* traj_turn_off,
     int32_t n_traj, int32_t n_turns, int64_t row_begin, int64_t row_end, int32_t stop_mode,
     const float* lambda, float lambda_all, stride_scan_state* state, const stride_row_outputs* out,
-    stride_turn_stats* turn_stats, int32_t* dev_status, void* stream) {
+    stride_turn_stats* turn_stats, double* profile, int32_t* dev_status, void* stream) {
   if (row_begin < 0 || row_end < row_begin) return STRIDE_ERR_INVALID_ARG;
   if (row_end - row_begin > (int64_t)STRIDE_NOALLOC_MAX_ROWS) return STRIDE_ERR_TOO_LARGE;
   if (row_end == row_begin) return STRIDE_OK;
@@ -88,5 +88,6 @@ extern "C" STRIDE_API int stride_score_batch_noalloc(
   // launches the kernel with pointers into the scratch.
   return stride_score_batch(S, T, dtype, ld, V, tokens, traj_row_off, turn_row_off, traj_turn_off,
                             n_traj, n_turns, row_begin, row_end, stop_mode, lambda, lambda_all,
-                            state, out, turn_stats, dev_status, scratch, kNoAllocBytes, stream);
+                            state, out, turn_stats, profile, dev_status, scratch, kNoAllocBytes,
+                            stream);
 }

@@ -81,6 +81,7 @@ struct alignas(128) StreamShared {
   float red[kSlots][kConsumerWarps][4];
   RowMeta slot_meta[kSlots];
   RowCarry slot_carry[kSlots];
+  double prof[3 * STRIDE_PROFILE_BINS];  // this CTA's within-turn profile (row warp only)
   int64_t end_seq;  // first row sequence number without a row (set by the row warp)
   int32_t abort;
 };
@@ -124,6 +125,7 @@ __global__ void __launch_bounds__(kStreamThreads, 1) score_batch_stream_kernel(c
     }
     sh.abort = 0;
     sh.end_seq = INT64_MAX;
+    for (int i = 0; i < 3 * STRIDE_PROFILE_BINS; ++i) sh.prof[i] = 0.0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
   __syncthreads();
@@ -327,12 +329,17 @@ __global__ void __launch_bounds__(kStreamThreads, 1) score_batch_stream_kernel(c
       lse_merge(mS, sS, tmS, tsS);
       lse_merge(mT, sT, tmT, tsT);
       if (lane == 0) {
-        sh.slot_carry[q] = row_finalize(p, tile, r, meta, y, xs, xt, lse_finish(mS, sS), lse_finish(mT, sT));
+        sh.slot_carry[q] = row_finalize(p, tile, r, meta, y, xs, xt, lse_finish(mS, sS), lse_finish(mT, sT),
+                                        p.profile ? sh.prof : nullptr, false);
         sh.slot_meta[q] = meta;
         mbar_arrive(&sh.agg_ready[q]);
       }
       __syncwarp();
       ++seq;
+    }
+    if (lane == 0 && p.profile) {
+      for (int i = 0; i < 3 * STRIDE_PROFILE_BINS; ++i)
+        if (sh.prof[i] != 0.0) atomicAdd(p.profile + i, sh.prof[i]);
     }
     return;
   }

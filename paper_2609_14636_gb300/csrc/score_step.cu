@@ -78,7 +78,7 @@ __global__ void __cluster_dims__(kStepCluster, 1, 1) __launch_bounds__(kStepThre
       if (o.x_s) o.x_s[b] = nan;
       if (o.x_t) o.x_t[b] = nan;
       if (p.stopped_now) p.stopped_now[b] = 0;
-      if (p.turn_out) p.turn_out[b] = stride_turn_stats{0.0, 0.0, 0.0, 0.f, 0};
+      if (p.turn_out) p.turn_out[b] = stride_turn_stats{0.0, 0.0, 0.0, 0.0, 0.f, 0};
     }
     return;
   }
@@ -167,8 +167,12 @@ __global__ void __cluster_dims__(kStepCluster, 1, 1) __launch_bounds__(kStepThre
       // carried state (Algorithm 1 inner loop)
       stride_scan_state st = *sp;
       const float lam = p.lambda ? __ldg(p.lambda + b) : p.lambda_all;
+      const double term = (double)lps * (double)dd;  // -log pi_S * r_t (Eq. 2); every scored token is retained
       st.turn_sum_t += (double)lpt;
       st.turn_sum_d += (double)dd;
+      st.turn_sum_l += term;
+      st.loss += term;
+      st.loss_tokens += 1;
       st.turn_tokens += 1;
       const int64_t pos = st.rows_seen;
       st.rows_seen += 1;
@@ -177,7 +181,7 @@ __global__ void __cluster_dims__(kStepCluster, 1, 1) __launch_bounds__(kStepThre
         st.cum += (double)lpt;
         if (st.cum < (double)lam) fired = 1;
       }
-      stride_turn_stats ts{0.0, 0.0, 0.0, 0.f, 0};
+      stride_turn_stats ts{0.0, 0.0, 0.0, 0.0, 0.f, 0};
       if (__ldg(p.turn_end + b)) {
         const double mean = st.turn_sum_t / (double)st.turn_tokens;  // Eq. 4
         if (p.mode == STRIDE_STOP_TURN_MEAN) {
@@ -186,6 +190,7 @@ __global__ void __cluster_dims__(kStepCluster, 1, 1) __launch_bounds__(kStepThre
         }
         ts.sum_t = st.turn_sum_t;
         ts.sum_d = st.turn_sum_d;
+        ts.sum_l = st.turn_sum_l;
         ts.cum = st.cum;
         ts.mean_t = (float)mean;
         ts.n = st.turn_tokens;
@@ -193,6 +198,7 @@ __global__ void __cluster_dims__(kStepCluster, 1, 1) __launch_bounds__(kStepThre
         st.turn_tokens = 0;
         st.turn_sum_t = 0.0;
         st.turn_sum_d = 0.0;
+        st.turn_sum_l = 0.0;
       }
       if (fired) {
         st.stopped = 1;

@@ -69,7 +69,10 @@ __global__ void state_init_kernel(stride_scan_state* s, int32_t n) {
   z.cum = 0.0;
   z.turn_sum_t = 0.0;
   z.turn_sum_d = 0.0;
+  z.turn_sum_l = 0.0;
+  z.loss = 0.0;
   z.rows_seen = 0;
+  z.loss_tokens = 0;
   z.stop_row = -1;
   z.stop_turn = -1;
   z.turn_tokens = 0;

@@ -10,9 +10,10 @@
 
 namespace stride {
 
-// One published scan element of the batch kernel's lookback (32 bytes).
+// One published scan element of the batch kernel's lookback (32 bytes):
+// running-sum terms, and the open turn's sums of log pi_T, d and logp_S * d.
 struct alignas(32) ScanSlot {
-  double c, st, sd, pad;
+  double c, st, sd, sl;
 };
 
 struct BatchParams {
@@ -35,6 +36,7 @@ struct BatchParams {
   stride_scan_state* state;
   stride_row_outputs out;
   stride_turn_stats* turn_stats;
+  double* profile;  // [STRIDE_PROFILE_BINS * 3] or NULL, added to
   int32_t* dev_status;
   // workspace views
   uint32_t* ticket;

@@ -11,6 +11,11 @@ Tolerances (stated where the path's outputs are specified):
   order -5; for sum_d, whose terms can cancel, the "+1" per token bounds the
   fp32 rounding of each d_i);
 * l_k (fp32): 2e-3 absolute (a mean of per-token values, each within 2e-3);
+* the OPD-loss sums (per turn, per trajectory over retained tokens):
+  1e-5 * sum(|logp_S * d| + |logp_S| + |d| + 1) over the summed tokens -- a
+  term logp_S * d carries the error of each factor scaled by the other;
+  the within-turn profile sums: like the per-turn sums; retained-token counts
+  and profile counts exact;
 * a stop index may differ from the oracle's only where the oracle's running
   sum lies within 1e-3 of lambda at every test position between the two.
 """
@@ -52,6 +57,7 @@ def run_batch(stride, S, T, tokens, lay, mode, lam, windows=None, V=None, out_ke
     offs = [torch.from_numpy(a).to(device) for a in (lay.traj_row_off, lay.turn_row_off, lay.traj_turn_off)]
     st = stride.new_state(lay.n_traj, device) if state is None else state
     ts = stride.new_turn_stats(lay.n_turns, device)
+    prof = stride.new_profile(device)
     keys = out_keys or stride.ROW_OUTPUT_KEYS
     out = {k: torch.full((R,), float("nan"), dtype=torch.float32, device=device) for k in keys}
     status = torch.zeros(1, dtype=torch.int32, device=device)
@@ -68,12 +74,13 @@ def run_batch(stride, S, T, tokens, lay, mode, lam, windows=None, V=None, out_ke
         o = {k: v[a - base:b - base] for k, v in out.items()}
         stride.stride_score_batch(St[a - base:b - base], Tt[a - base:b - base], tk[a - base:b - base], *offs,
                                   a, b, mode, lam_arg, st, out=o, turn_stats=ts, dev_status=status,
-                                  workspace=ws, V=V)
+                                  workspace=ws, V=V, profile=prof)
     torch.cuda.synchronize()
     res = {k: v.cpu().numpy() for k, v in out.items()}
     res["state"] = stride.state_to_numpy(st)[: lay.n_traj]
     res["turn_stats"] = stride.turn_stats_to_numpy(ts)[: lay.n_turns]
     res["status"] = int(status.item())
+    res["profile"] = prof.cpu().numpy()
     return res
 
 
@@ -81,9 +88,15 @@ def oracle_batch(S, T, tokens, lay, mode, lam, V=None):
     o = oracle.row_logprobs(S, T, tokens, V=V, check=False)
     lam64 = np.asarray(lam, np.float32).astype(np.float64)
     sc = oracle.scan_batch(o["logp_t"], o["d"], lay.traj_row_off, lay.turn_row_off, lay.traj_turn_off,
-                           mode, lam64)
+                           mode, lam64, logp_s=o["logp_s"])
     o.update(sc)
     return o
+
+
+def loss_mag(ls, d) -> float:
+    """Magnitude a sum of OPD-loss terms logp_S * d is compared against."""
+    ls, d = np.asarray(ls, np.float64), np.asarray(d, np.float64)
+    return float(np.sum(np.abs(ls * d) + np.abs(ls) + np.abs(d) + 1.0))
 
 
 def stop_matches(g_row, o_row, rc, tests, lam):
@@ -127,6 +140,8 @@ def compare_scan(g, o, lay, mode, lam):
         mag_d = np.sum(np.abs(d[a:b]) + 1.0)
         assert abs(ts["sum_t"][k] - o["turn_sum_t"][k]) <= SUM_RTOL * mag_t, ("sum_t", k)
         assert abs(ts["sum_d"][k] - o["turn_sum_d"][k]) <= SUM_RTOL * mag_d, ("sum_d", k)
+        mag_l = loss_mag(lp[a:b] + d[a:b], d[a:b])
+        assert abs(ts["sum_l"][k] - o["turn_sum_l"][k]) <= SUM_RTOL * mag_l, ("sum_l", k)
         assert abs(ts["mean_t"][k] - o["turn_mean"][k]) <= LOGP_ATOL, ("mean_t", k)
         assert abs(ts["cum"][k] - o["turn_cum"][k]) <= SUM_RTOL * abs(o["turn_cum"][k]) + 1e-12, ("cum", k)
     st = g["state"]
@@ -149,6 +164,17 @@ def compare_scan(g, o, lay, mode, lam):
             assert int(st["stop_turn"][i]) == int(o["stop_turn"][i]), (i, st["stop_turn"][i], o["stop_turn"][i])
         assert bool(st["stopped"][i]) == (gr >= 0)
         assert int(st["rows_seen"][i]) == r1 - r0
+        if gr == orr:
+            # OPD loss on the retained tokens (Eq. 2, Algorithm 1)
+            assert int(st["loss_tokens"][i]) == int(o["traj_loss_tokens"][i]), ("loss_tokens", i)
+            mag = loss_mag(lp[r0:r1] + d[r0:r1], d[r0:r1])
+            assert abs(st["loss"][i] - o["traj_loss"][i]) <= SUM_RTOL * mag, ("loss", i)
+    if "profile" in g:
+        # within-turn decile profile (Observation 1): counts exact, sums 1e-5 of magnitudes
+        gp, op = g["profile"], o["profile"]
+        assert np.array_equal(gp[:, 2], op[:, 2]), (gp[:, 2], op[:, 2])
+        assert np.all(np.abs(gp[:, 0] - op[:, 0]) <= SUM_RTOL * (np.sum(np.abs(d)) + len(d))), "profile d"
+        assert np.all(np.abs(gp[:, 1] - op[:, 1]) <= SUM_RTOL * np.sum(np.abs(lp) + 1.0)), "profile logp_t"
 
 
 def pad_cols(a: np.ndarray, ld: int, fill) -> np.ndarray:

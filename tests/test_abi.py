@@ -37,7 +37,7 @@ def test_library_exports_declared_symbols():
 def test_host_only_calls():
     import paper_2609_14636_gb300 as stride
 
-    assert stride.stride_abi_version() == 1
+    assert stride.stride_abi_version() == 2
     assert stride.stride_score_batch_workspace_size(0) == 0
     assert stride.stride_score_batch_workspace_size(1000) >= 1000 * 68
     assert "INVALID_ARG" in stride.stride_status_string(1)
@@ -46,6 +46,6 @@ def test_host_only_calls():
 def test_header_compiles_as_c():
     pytest.importorskip("subprocess")
     r = subprocess.run(["gcc", "-std=c99", "-Wall", "-Werror", "-fsyntax-only", "-x", "c", "-I", str(ROOT / "include"), "-"],
-                       input='#include "stride.h"\n#include "stride_selftest.h"\nint main(void){return sizeof(stride_scan_state)==56 && sizeof(stride_turn_stats)==32 ? 0 : 1;}\n',
+                       input='#include "stride.h"\n#include "stride_selftest.h"\nint main(void){return sizeof(stride_scan_state)==80 && sizeof(stride_turn_stats)==40 ? 0 : 1;}\n',
                        capture_output=True, text=True)
     assert r.returncode == 0, r.stderr

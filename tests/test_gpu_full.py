@@ -73,6 +73,7 @@ def stream_and_score(stride, w, lam, chunk_rows, resident=False):
     offs = [torch.from_numpy(a).to(dev) for a in (lay.traj_row_off, lay.turn_row_off, lay.traj_turn_off)]
     st = stride.new_state(lay.n_traj)
     ts = stride.new_turn_stats(lay.n_turns)
+    prof = stride.new_profile(dev)
     status = torch.zeros(1, dtype=torch.int32, device=dev)
     keys = stride.ROW_OUTPUT_KEYS
     g = {k: np.empty(R, np.float32) for k in keys}
@@ -93,7 +94,7 @@ def stream_and_score(stride, w, lam, chunk_rows, resident=False):
             synth.generate_rows(w.recipe, a + c, d - c, device=dev, out_S=S[c:d], out_T=T[c:d], out_tok=tok[c:d])
         stride.stride_score_batch(S[:n], T[:n], tok[:n], *offs, a, b, stride.TURN_MEAN, float(lam), st,
                                   out={k: v[:n] for k, v in out.items()}, turn_stats=ts, dev_status=status,
-                                  workspace=ws)
+                                  workspace=ws, profile=prof)
         torch.cuda.synchronize()
         for k in keys:
             g[k][a:b] = out[k][:n].cpu().numpy()
@@ -101,8 +102,9 @@ def stream_and_score(stride, w, lam, chunk_rows, resident=False):
     g["state"] = stride.state_to_numpy(st)[: lay.n_traj]
     g["turn_stats"] = stride.turn_stats_to_numpy(ts)[: lay.n_turns]
     g["status"] = int(status.item())
+    g["profile"] = prof.cpu().numpy()
     sc = oracle.scan_batch(o["logp_t"], o["d"], lay.traj_row_off, lay.turn_row_off, lay.traj_turn_off,
-                           oracle.TURN_MEAN, float(np.float32(lam)))
+                           oracle.TURN_MEAN, float(np.float32(lam)), logp_s=o["logp_s"])
     o.update(sc)
     return g, o
 

@@ -7,7 +7,7 @@ import pytest
 
 import oracle
 import synth
-from gpu_helpers import LOGP_ATOL, SUM_RTOL, TIE_BAND, to_dev
+from gpu_helpers import LOGP_ATOL, SUM_RTOL, TIE_BAND, loss_mag, to_dev
 
 pytestmark = pytest.mark.gpu
 
@@ -41,11 +41,13 @@ def run_steps(stride, St, Tt, tk, turn_end, ring, B, mode, lam, V, check_every=N
     te_dev = torch.from_numpy(turn_end).cuda()
     out = {k: torch.empty(B, dtype=torch.float32, device="cuda") for k in ("logp_s", "logp_t", "opd")}
     sn = torch.empty(B, dtype=torch.uint8, device="cuda")
-    tout = torch.empty((B, 32), dtype=torch.uint8, device="cuda")
+    tout = torch.empty((B, stride.TURN_STATS_DTYPE.itemsize), dtype=torch.uint8, device="cuda")
     lam_arg = float(np.float32(lam))
     fired_g = np.zeros((steps, B), np.uint8)
     fired_o = np.zeros((steps, B), np.uint8)
     worst = 0.0
+    loss_m = np.zeros(B)        # magnitude of each rollout's loss sum so far
+    turn_m = np.zeros(B)        # ... of its open turn's loss sum
     for s in range(steps):
         j = s % ring
         stride.stride_score_step(St[j * B:(j + 1) * B], Tt[j * B:(j + 1) * B], tk[j * B:(j + 1) * B], te_dev[s],
@@ -53,6 +55,12 @@ def run_steps(stride, St, Tt, tk, turn_end, ring, B, mode, lam, V, check_every=N
         ps, pt = o_rows["logp_s"][j * B:(j + 1) * B], o_rows["logp_t"][j * B:(j + 1) * B]
         oo = oracle.step_update(ost, ps, pt, turn_end[s], mode, np.float32(lam))
         fired_o[s] = oo["stopped_now"]
+        act_now = ~np.isnan(oo["logp_t"])
+        m_now = np.where(act_now, np.abs(ps * (ps - pt)) + np.abs(ps) + np.abs(ps - pt) + 1.0, 0.0)
+        loss_m += m_now
+        turn_m += m_now
+        closed_mag = turn_m.copy()
+        turn_m[oo["turn_n"] > 0] = 0.0
         if check_every and (s % check_every == 0 or s == steps - 1):
             torch.cuda.synchronize()
             g_lp = out["logp_t"].cpu().numpy()
@@ -66,8 +74,11 @@ def run_steps(stride, St, Tt, tk, turn_end, ring, B, mode, lam, V, check_every=N
             assert np.array_equal(tg["n"], oo["turn_n"])
             if closed.any():
                 assert np.all(np.abs(tg["mean_t"][closed] - oo["turn_mean"][closed]) <= LOGP_ATOL)
+                assert np.all(np.abs(tg["sum_l"][closed] - oo["turn_sum_l"][closed]) <= SUM_RTOL * closed_mag[closed])
     torch.cuda.synchronize()
-    return stride.state_to_numpy(st), oracle.rollouts_to_numpy(ost), worst
+    o = oracle.rollouts_to_numpy(ost)
+    o["loss_mag"] = loss_m
+    return stride.state_to_numpy(st), o, worst
 
 
 def _check_final(g, o, mode, lam):
@@ -81,6 +92,8 @@ def _check_final(g, o, mode, lam):
         assert g["rows_seen"][b] == o["rows_seen"][b]
         assert g["turn_idx"][b] == o["turn_idx"][b] and g["turn_tokens"][b] == o["turn_tokens"][b]
         assert abs(g["cum"][b] - o["cum"][b]) <= SUM_RTOL * abs(o["cum"][b]) + 1e-12
+        assert g["loss_tokens"][b] == g["rows_seen"][b]
+        assert abs(g["loss"][b] - o["loss"][b]) <= SUM_RTOL * o["loss_mag"][b]
 
 
 @pytest.mark.parametrize("mode,lam", [(0, -30.0), (1, -400.0)])

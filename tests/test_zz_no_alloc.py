@@ -62,8 +62,9 @@ def _same(a, b):
     for f in ("sum_t", "cum"):
         x, y = a["turn_stats"][f], b["turn_stats"][f]
         assert np.all(np.abs(x - y) <= SUM_RTOL * np.abs(y) + 1e-12), f
-    for f in ("stop_row", "stop_turn", "rows_seen", "stopped"):
+    for f in ("stop_row", "stop_turn", "rows_seen", "stopped", "loss_tokens"):
         assert np.array_equal(a["state"][f], b["state"][f]), f
+    assert np.all(np.abs(a["state"]["loss"] - b["state"]["loss"]) <= SUM_RTOL * (np.abs(b["state"]["loss"]) + 1.0))
     assert np.all(np.abs(a["state"]["cum"] - b["state"]["cum"]) <= SUM_RTOL * np.abs(b["state"]["cum"]))
 
 
