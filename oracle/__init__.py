@@ -14,6 +14,8 @@ marshals numpy arrays.  Definitions followed (see the C file for detail):
   prefix-buffer offset (Sec. 4.1), token-level variant (Sec. 5.5).
 * :func:`step_update`    -- Algorithm 1's inner loop, one token per call.
 * :func:`select_restart` -- quality gate (Sec. 4.2), K_max, Eq. 6.
+* :func:`buffer_record`  -- Algorithm 1's record of {l_k} in H(x), with the
+  reused prefix kept (Sec. 4.2 step 3).
 """
 from __future__ import annotations
 
@@ -65,6 +67,8 @@ class OracleLib:
         lib.oracle_select_restart.argtypes = [P, P, P, ctypes.c_float, i32, i32, P, P]
         lib.oracle_select_restart.restype = ci
         lib.oracle_rollout_size.restype = ci
+        lib.oracle_buffer_record.argtypes = [P, P, i32, i32, P, P, P, P, i32]
+        lib.oracle_buffer_record.restype = ci
         self.lib = lib
 
     # ---- Eq. 1 / Eq. 4: per-row log-probs --------------------------------
@@ -168,6 +172,21 @@ class OracleLib:
             raise ValueError(f"oracle_step_update returned {rc}")
         return out
 
+    # ---- Algorithm 1: record {l_k} to H(x) ----------------------------------
+    def buffer_record(self, mean, n_turns, task, k0, turn_mean, traj_turn_off):
+        """Update a prefix buffer in place (numpy arrays mean [n_tasks, T_max]
+        float32 and n_turns [n_tasks] int32) with the trajectories' records."""
+        assert mean.dtype == np.float32 and mean.flags.c_contiguous and n_turns.dtype == np.int32
+        n_tasks, T_max = mean.shape
+        tk = np.ascontiguousarray(task, np.int32)
+        k0a = None if k0 is None else np.ascontiguousarray(k0, np.int32)
+        tm = np.ascontiguousarray(turn_mean, np.float32)
+        tto = np.ascontiguousarray(traj_turn_off, np.int32)
+        rc = self.lib.oracle_buffer_record(_ptr(mean), _ptr(n_turns), n_tasks, T_max, _ptr(tk), _ptr(k0a),
+                                           _ptr(tm), _ptr(tto), tk.shape[0])
+        if rc != OK:
+            raise ValueError(f"oracle_buffer_record returned {rc}")
+
     # ---- Sec. 4.2 / Eq. 6: restart choice -----------------------------------
     def select_restart(self, mean, n_turns, mask, alpha: float):
         """Quality gate, K_max and the weakest correct turn.  Returns
@@ -242,3 +261,7 @@ def step_update(*a, **k):
 
 def select_restart(*a, **k):
     return get().select_restart(*a, **k)
+
+
+def buffer_record(*a, **k):
+    return get().buffer_record(*a, **k)

@@ -429,4 +429,32 @@ int oracle_select_restart(const float* mean, const int32_t* n_turns, const uint8
   return ORACLE_OK;
 }
 
+/* Prefix buffer update (Algorithm 1: "record this trajectory's {l_k} to
+ * H(x)"; Sec. 4.2 step 3, prefix reuse).  Trajectory i belongs to task
+ * task[i] and reused the first k0[i] turns of that task's stored record as
+ * context, so its own record is those k0[i] stored turns followed by the
+ * means of its newly generated turns (turn_mean over its turns
+ * traj_turn_off[i] .. traj_turn_off[i+1]-1, stored in fp32), truncated to
+ * T_max turns.  k0[i] is clamped to the stored record's length.  Each task
+ * may appear at most once per call.  mean: [n_tasks, T_max]; n_turns:
+ * [n_tasks]. */
+int oracle_buffer_record(float* mean, int32_t* n_turns, int32_t n_tasks, int32_t T_max,
+                         const int32_t* task, const int32_t* k0, const float* turn_mean,
+                         const int32_t* traj_turn_off, int32_t n_traj) {
+  if (!mean || !n_turns || !task || !turn_mean || !traj_turn_off || n_traj < 0 || T_max < 0)
+    return ORACLE_ERR_ARG;
+  for (int32_t i = 0; i < n_traj; ++i) {
+    int32_t x = task[i];
+    if (x < 0 || x >= n_tasks) return ORACLE_ERR_ARG;
+    int32_t keep = k0 ? k0[i] : 0;
+    if (keep < 0) keep = 0;
+    if (keep > n_turns[x]) keep = n_turns[x];
+    int32_t len = keep;
+    for (int32_t k = traj_turn_off[i]; k < traj_turn_off[i + 1] && len < T_max; ++k)
+      mean[(int64_t)x * T_max + len++] = turn_mean[k];
+    n_turns[x] = len;
+  }
+  return ORACLE_OK;
+}
+
 int oracle_rollout_size(void) { return (int)sizeof(oracle_rollout); }

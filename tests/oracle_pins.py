@@ -496,6 +496,48 @@ def check_select_bruteforce(orc):
             assert km[i] == K and ks[i] == kstar, (i, alpha)
 
 
+def check_prefix_buffer_golden(orc):
+    """Algorithm 1's record of {l_k} in H(x) with the reused prefix kept, and
+    the restart choice before and after (hand-worked cases)."""
+    cases = json.loads((GOLD / "prefix_buffer_cases.json").read_text())["cases"]
+    for c in cases:
+        T_max = c["T_max"]
+        mean = np.full((1, T_max), np.float32(123.0), np.float32)
+        n = np.array([len(c["stored"])], np.int32)
+        mean[0, :len(c["stored"])] = c["stored"]
+        ks, km = orc.select_restart(mean, n, None, _f(c["alpha"]))
+        assert (int(km[0]), int(ks[0])) == (c["select_before"]["k_max"], c["select_before"]["k_star"]), c["name"]
+        new = np.array(c["new_turn_means"], np.float32)
+        orc.buffer_record(mean, n, [0], ks, new, [0, len(new)])
+        assert int(n[0]) == len(c["record_after"]), c["name"]
+        assert list(mean[0, :n[0]]) == c["record_after"], (c["name"], mean[0, :n[0]])
+        ks, km = orc.select_restart(mean, n, None, _f(c["alpha"]))
+        assert (int(km[0]), int(ks[0])) == (c["select_after"]["k_max"], c["select_after"]["k_star"]), c["name"]
+
+
+def check_prefix_buffer_properties(orc):
+    """Random records: the kept prefix is unchanged, the new means follow it,
+    k0 beyond the stored length is clamped, other tasks are untouched."""
+    rng = np.random.default_rng(31)
+    n_tasks, T_max = 40, 9
+    mean = rng.standard_normal((n_tasks, T_max)).astype(np.float32)
+    n = rng.integers(0, T_max + 1, n_tasks).astype(np.int32)
+    before_m, before_n = mean.copy(), n.copy()
+    tasks = rng.permutation(n_tasks)[:25].astype(np.int32)
+    k0 = rng.integers(0, T_max + 3, 25).astype(np.int32)
+    lens = rng.integers(0, 7, 25)
+    off = np.concatenate([[0], np.cumsum(lens)]).astype(np.int32)
+    tm = rng.standard_normal(int(off[-1])).astype(np.float32)
+    orc.buffer_record(mean, n, tasks, k0, tm, off)
+    for j, x in enumerate(tasks):
+        keep = min(int(k0[j]), int(before_n[x]))
+        want = np.concatenate([before_m[x, :keep], tm[off[j]:off[j + 1]]])[:T_max]
+        assert int(n[x]) == len(want)
+        assert np.array_equal(mean[x, :n[x]], want)
+    others = np.setdiff1d(np.arange(n_tasks), tasks)
+    assert np.array_equal(mean[others], before_m[others]) and np.array_equal(n[others], before_n[others])
+
+
 ALL_CHECKS = [
     check_uniform_closed_form, check_one_hot_closed_form, check_d_sign_and_operands,
     check_bruteforce_mpmath, check_normalisation, check_shift_invariance, check_torch_log_softmax,
@@ -505,4 +547,5 @@ ALL_CHECKS = [
     check_opd_loss_golden, check_turn_profile_golden, check_loss_invariants,
     check_step_matches_batch, check_step_golden,
     check_select_golden, check_select_bruteforce,
+    check_prefix_buffer_golden, check_prefix_buffer_properties,
 ]

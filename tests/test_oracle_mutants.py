@@ -45,6 +45,9 @@ MUTANTS = [
      "if (st_row < 0 && cum + lt >= lambda[i]) {\n            loss += term;"),
     ("profile_wrong_decile", "int64_t j = (10 * (r - a)) / n;", "int64_t j = (10 * (r - a)) / (n + 1);"),
     ("step_loss_teacher", "s->loss += ps * dd;", "s->loss += pt * dd;"),
+    ("record_drops_prefix", "int32_t len = keep;", "int32_t len = 0;"),
+    ("record_no_clamp", "if (keep > n_turns[x]) keep = n_turns[x];", "if (keep > T_max) keep = T_max;"),
+    ("record_prefix_off_by_one", "int32_t keep = k0 ? k0[i] : 0;", "int32_t keep = k0 ? k0[i] + 1 : 0;"),
 ]
 
 
