@@ -270,6 +270,26 @@ STRIDE_API int stride_score_batch_noalloc(const void* S, const void* T, int32_t 
                                           stride_turn_stats* turn_stats, double* profile,
                                           int32_t* dev_status, void* stream);
 
+/* Record trajectories in a device-resident prefix buffer H(x) (Algorithm 1:
+ * "record this trajectory's {l_k} to H(x)"; Sec. 4.2 step 3, prefix reuse).
+ *
+ * buf_mean: float [n_tasks, T_max] and buf_n_turns: int32 [n_tasks], the
+ * buffer, updated in place (the same layout stride_select_restart reads, so
+ * score -> record -> select runs on the device).  Trajectory i belongs to
+ * task task_of_traj[i] (int32 [n_traj]) and reused the first k0_of_traj[i]
+ * turns of that task's stored record as context (int32 [n_traj], the k* the
+ * previous select returned; NULL = 0 for all); its record becomes those
+ * stored turns followed by the l_k (turn_stats[k].mean_t) of its own turns
+ * traj_turn_off[i] .. traj_turn_off[i+1]-1, truncated to T_max.  k0 is
+ * clamped to the stored length.  Each task may appear at most once per call
+ * (otherwise the records of the duplicates race).  A task id outside
+ * [0, n_tasks) sets STRIDE_DEV_BAD_LAYOUT and that trajectory is skipped. */
+STRIDE_API int stride_buffer_record(float* buf_mean, int32_t* buf_n_turns, int32_t n_tasks,
+                                    int32_t T_max, const int32_t* task_of_traj,
+                                    const int32_t* k0_of_traj, const stride_turn_stats* turn_stats,
+                                    const int32_t* traj_turn_off, int32_t n_traj,
+                                    int32_t* dev_status, void* stream);
+
 /* Human-readable name of a stride_status code (static string). */
 STRIDE_API const char* stride_status_string(int code);
 

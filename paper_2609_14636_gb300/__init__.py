@@ -29,7 +29,7 @@ __all__ = [
     "stride_score_batch_workspace_size", "stride_score_batch", "stride_score_step",
     "stride_select_restart", "stride_status_string", "stride_abi_version", "ROW_OUTPUT_KEYS",
     "stride_score_batch_noalloc", "NOALLOC_MAX_ROWS", "ERR_TOO_LARGE", "PROFILE_BINS", "new_profile",
-    "stride_selftest_bounded_wait",
+    "stride_selftest_bounded_wait", "stride_buffer_record",
 ]
 
 DTYPE_BF16, DTYPE_F32 = 0, 1
@@ -80,6 +80,8 @@ def lib() -> ctypes.CDLL:
                                          P, P, P, P, P, P, sz, P]
         L.stride_score_step.argtypes = [P, P, i32, i64, i64, P, P, i32, i32, P, f32, P, P, P, P, P, P]
         L.stride_select_restart.argtypes = [P, P, P, f32, i32, i32, P, P, P]
+        L.stride_buffer_record.argtypes = [P, P, i32, i32, P, P, P, P, i32, P, P]
+        L.stride_buffer_record.restype = ctypes.c_int
         L.stride_selftest_bounded_wait.argtypes = [i32, ctypes.c_uint64, P, P, sz, P]
         L.stride_selftest_bounded_wait.restype = ctypes.c_int
         L.stride_score_batch_noalloc.argtypes = [P, P, i32, i64, i64, P, P, P, P, i32, i32, i64, i64, i32,
@@ -286,6 +288,25 @@ def stride_select_restart(turn_mean, n_turns, correct, alpha: float, k_star, k_m
         _dev(correct, "correct", torch.uint8, N * T_max, optional=True), float(alpha), N, T_max,
         _dev(k_star, "k_star", torch.int32, N), _dev(k_max, "k_max", torch.int32, N), _stream(stream))
     _check("stride_select_restart", rc)
+
+
+def stride_buffer_record(buf_mean, buf_n_turns, task_of_traj, k0_of_traj, turn_stats, traj_turn_off,
+                         dev_status=None, stream=None) -> None:
+    """Record trajectories' turn means in the prefix buffer H(x) (float32
+    [n_tasks, T_max] and int32 [n_tasks], updated in place): each keeps the
+    first k0 stored turns of its task, then its own turns (Algorithm 1)."""
+    torch = _torch()
+    if buf_mean.dim() != 2:
+        raise ValueError("buf_mean must be [n_tasks, T_max]")
+    n_tasks, T_max = buf_mean.shape
+    n_traj = traj_turn_off.numel() - 1
+    rc = lib().stride_buffer_record(
+        _dev(buf_mean, "buf_mean", torch.float32), _dev(buf_n_turns, "buf_n_turns", torch.int32, n_tasks),
+        n_tasks, T_max, _dev(task_of_traj, "task_of_traj", torch.int32, n_traj),
+        _dev(k0_of_traj, "k0_of_traj", torch.int32, n_traj, optional=True),
+        _dev(turn_stats, "turn_stats", torch.uint8), _dev(traj_turn_off, "traj_turn_off", torch.int32, n_traj + 1),
+        n_traj, _dev(dev_status, "dev_status", torch.int32, 1, optional=True), _stream(stream))
+    _check("stride_buffer_record", rc)
 
 
 SELFTEST_LOOKBACK, SELFTEST_MBARRIER = 0, 1

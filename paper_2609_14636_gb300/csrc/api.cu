@@ -209,4 +209,21 @@ int stride_select_restart(const float* turn_mean, const int32_t* n_turns, const 
                                                                               : STRIDE_ERR_CUDA;
 }
 
+int stride_buffer_record(float* buf_mean, int32_t* buf_n_turns, int32_t n_tasks, int32_t T_max,
+                         const int32_t* task_of_traj, const int32_t* k0_of_traj,
+                         const stride_turn_stats* turn_stats, const int32_t* traj_turn_off,
+                         int32_t n_traj, int32_t* dev_status, void* stream) {
+  if (n_traj < 0 || n_tasks < 0 || T_max < 0) return STRIDE_ERR_INVALID_ARG;
+  if (n_traj == 0) return STRIDE_OK;
+  if (!buf_mean || !buf_n_turns || !task_of_traj || !turn_stats || !traj_turn_off)
+    return STRIDE_ERR_INVALID_ARG;
+  const int dc = check_device();
+  if (dc != STRIDE_OK) return dc;
+  return stride::launch_buffer_record(buf_mean, buf_n_turns, n_tasks, T_max, task_of_traj, k0_of_traj,
+                                      turn_stats, traj_turn_off, n_traj, dev_status,
+                                      (cudaStream_t)stream) == cudaSuccess
+             ? STRIDE_OK
+             : STRIDE_ERR_CUDA;
+}
+
 }  // extern "C"

@@ -62,6 +62,31 @@ __global__ void __launch_bounds__(kSelectThreads) select_restart_kernel(const Se
   }
 }
 
+// One warp per trajectory: keep the task's first k0 stored turns, append the
+// trajectory's turn means, set the record length (Algorithm 1, record step).
+__global__ void __launch_bounds__(kSelectThreads) buffer_record_kernel(
+    float* buf_mean, int32_t* buf_n_turns, int32_t n_tasks, int32_t T_max, const int32_t* task,
+    const int32_t* k0, const stride_turn_stats* ts, const int32_t* traj_turn_off, int32_t n_traj,
+    int32_t* dev_status) {
+  const int lane = threadIdx.x & 31;
+  const int64_t i = ((int64_t)blockIdx.x * kSelectThreads + threadIdx.x) >> 5;
+  if (i >= n_traj) return;
+  const int32_t x = __ldg(task + i);
+  if (x < 0 || x >= n_tasks) {
+    if (lane == 0) set_status(dev_status, STRIDE_DEV_BAD_LAYOUT);
+    return;
+  }
+  const int32_t stored = __ldg(buf_n_turns + x);
+  int32_t keep = k0 ? __ldg(k0 + i) : 0;
+  keep = keep < 0 ? 0 : (keep > stored ? stored : keep);
+  const int32_t a = __ldg(traj_turn_off + i), b = __ldg(traj_turn_off + i + 1);
+  const int32_t n_new = b > a ? b - a : 0;
+  const int32_t len = keep + n_new < T_max ? keep + n_new : (keep < T_max ? T_max : keep);
+  float* row = buf_mean + (int64_t)x * T_max;
+  for (int32_t j = keep + lane; j < len; j += 32) row[j] = ts[a + (j - keep)].mean_t;
+  if (lane == 0) buf_n_turns[x] = len;
+}
+
 __global__ void state_init_kernel(stride_scan_state* s, int32_t n) {
   const int32_t i = blockIdx.x * blockDim.x + threadIdx.x;
   if (i >= n) return;
@@ -85,6 +110,17 @@ cudaError_t launch_select_restart(const SelectParams& p, cudaStream_t stream) {
   const int64_t warps_per_block = kSelectThreads / 32;
   const unsigned grid = (unsigned)((p.N + warps_per_block - 1) / warps_per_block);
   select_restart_kernel<<<grid, kSelectThreads, 0, stream>>>(p);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_buffer_record(float* buf_mean, int32_t* buf_n_turns, int32_t n_tasks, int32_t T_max,
+                                 const int32_t* task, const int32_t* k0, const stride_turn_stats* ts,
+                                 const int32_t* traj_turn_off, int32_t n_traj, int32_t* dev_status,
+                                 cudaStream_t stream) {
+  const int64_t warps_per_block = kSelectThreads / 32;
+  const unsigned grid = (unsigned)((n_traj + warps_per_block - 1) / warps_per_block);
+  buffer_record_kernel<<<grid, kSelectThreads, 0, stream>>>(buf_mean, buf_n_turns, n_tasks, T_max, task, k0,
+                                                            ts, traj_turn_off, n_traj, dev_status);
   return cudaGetLastError();
 }
 

@@ -87,5 +87,9 @@ cudaError_t launch_score_batch_stream(const BatchParams& p, int dtype, cudaStrea
 cudaError_t launch_score_step(const StepParams& p, int dtype, bool vec, cudaStream_t stream);
 cudaError_t launch_select_restart(const SelectParams& p, cudaStream_t stream);
 cudaError_t launch_state_init(stride_scan_state* state, int32_t n, cudaStream_t stream);
+cudaError_t launch_buffer_record(float* buf_mean, int32_t* buf_n_turns, int32_t n_tasks, int32_t T_max,
+                                 const int32_t* task, const int32_t* k0, const stride_turn_stats* ts,
+                                 const int32_t* traj_turn_off, int32_t n_traj, int32_t* dev_status,
+                                 cudaStream_t stream);
 
 }  // namespace stride
