@@ -196,6 +196,30 @@ STRIDE_API int stride_score_batch(const void* S, const void* T, int32_t dtype, i
                        double* profile, int32_t* dev_status, void* workspace,
                        size_t workspace_bytes, void* stream);
 
+/* stride_score_batch with one teacher per domain, without gathering the
+ * teacher rows (Sec. 5.3: in cross-domain multi-teacher OPD each trajectory
+ * is scored by the expert teacher of its own domain).
+ *
+ * The student logits S are as in stride_score_batch (one row per window
+ * row).  The teacher logits of domain j live in their own buffer
+ * T_domains[j] ([T_domain_rows[j], ld_T] row-major, device; T_domains and
+ * T_domain_rows are HOST arrays of n_domains <= 8 entries).  Trajectory i is
+ * scored against domain traj_domain[i] (device uint8 [n_traj]); its rows are
+ * rows traj_T_row0[i], traj_T_row0[i]+1, ... of that buffer (device int64
+ * [n_traj]).  A domain or teacher row out of range sets
+ * STRIDE_DEV_BAD_LAYOUT (that row's results are meaningless; nothing faults).
+ * The workspace must hold stride_score_batch_workspace_size(rows) plus 8
+ * bytes per row (rounded up to 256).  All other arguments and results are
+ * those of stride_score_batch. */
+STRIDE_API int stride_score_batch_multi_teacher(
+    const void* S, const void* const* T_domains, const int64_t* T_domain_rows, int32_t n_domains,
+    int64_t ld_T, const uint8_t* traj_domain, const int64_t* traj_T_row0, int32_t dtype, int64_t ld,
+    int64_t V, const int32_t* tokens, const int64_t* traj_row_off, const int64_t* turn_row_off,
+    const int32_t* traj_turn_off, int32_t n_traj, int32_t n_turns, int64_t row_begin,
+    int64_t row_end, int32_t stop_mode, const float* lambda, float lambda_all,
+    stride_scan_state* state, const stride_row_outputs* out, stride_turn_stats* turn_stats,
+    double* profile, int32_t* dev_status, void* workspace, size_t workspace_bytes, void* stream);
+
 /* One decode step over B rollouts (Algorithm 1, inner turn loop, one
  * generated token per rollout).
  *

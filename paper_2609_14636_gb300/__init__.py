@@ -29,7 +29,8 @@ __all__ = [
     "stride_score_batch_workspace_size", "stride_score_batch", "stride_score_step",
     "stride_select_restart", "stride_status_string", "stride_abi_version", "ROW_OUTPUT_KEYS",
     "stride_score_batch_noalloc", "NOALLOC_MAX_ROWS", "ERR_TOO_LARGE", "PROFILE_BINS", "new_profile",
-    "stride_selftest_bounded_wait", "stride_buffer_record",
+    "stride_selftest_bounded_wait", "stride_buffer_record", "stride_score_batch_multi_teacher",
+    "multi_teacher_workspace_size",
 ]
 
 DTYPE_BF16, DTYPE_F32 = 0, 1
@@ -81,6 +82,9 @@ def lib() -> ctypes.CDLL:
         L.stride_score_step.argtypes = [P, P, i32, i64, i64, P, P, i32, i32, P, f32, P, P, P, P, P, P]
         L.stride_select_restart.argtypes = [P, P, P, f32, i32, i32, P, P, P]
         L.stride_buffer_record.argtypes = [P, P, i32, i32, P, P, P, P, i32, P, P]
+        L.stride_score_batch_multi_teacher.argtypes = [P, P, P, i32, i64, P, P, i32, i64, i64, P, P, P, P, i32,
+                                                       i32, i64, i64, i32, P, f32, P, P, P, P, P, P, sz, P]
+        L.stride_score_batch_multi_teacher.restype = ctypes.c_int
         L.stride_buffer_record.restype = ctypes.c_int
         L.stride_selftest_bounded_wait.argtypes = [i32, ctypes.c_uint64, P, P, sz, P]
         L.stride_selftest_bounded_wait.restype = ctypes.c_int
@@ -288,6 +292,57 @@ def stride_select_restart(turn_mean, n_turns, correct, alpha: float, k_star, k_m
         _dev(correct, "correct", torch.uint8, N * T_max, optional=True), float(alpha), N, T_max,
         _dev(k_star, "k_star", torch.int32, N), _dev(k_max, "k_max", torch.int32, N), _stream(stream))
     _check("stride_select_restart", rc)
+
+
+def multi_teacher_workspace_size(window_rows: int) -> int:
+    """Workspace bytes of stride_score_batch_multi_teacher for a window."""
+    return stride_score_batch_workspace_size(window_rows) + ((8 * int(window_rows) + 255) & ~255)
+
+
+def stride_score_batch_multi_teacher(S, T_domains, traj_domain, traj_T_row0, tokens, traj_row_off, turn_row_off,
+                                     traj_turn_off, row_begin: int, row_end: int, stop_mode: int, lam, state,
+                                     out: dict | None = None, turn_stats=None, dev_status=None, workspace=None,
+                                     V: int | None = None, stream=None, profile=None) -> None:
+    """Batch scoring with one teacher logit buffer per domain (list of 2-D
+    CUDA tensors of S's dtype and a common row stride), a per-trajectory
+    domain id (uint8) and the trajectory's first row in its domain buffer
+    (int64).  See include/stride.h."""
+    torch = _torch()
+    if not isinstance(S, torch.Tensor) or not S.is_cuda or S.dim() != 2 or S.stride(1) != 1:
+        raise TypeError("S must be a 2-D CUDA tensor with unit column stride")
+    if S.dtype == torch.bfloat16:
+        dt = DTYPE_BF16
+    elif S.dtype == torch.float32:
+        dt = DTYPE_F32
+    else:
+        raise TypeError(f"logits must be bfloat16 or float32, got {S.dtype}")
+    D = len(T_domains)
+    if D < 1:
+        raise ValueError("at least one teacher domain")
+    ld_T = T_domains[0].stride(0)
+    for t in T_domains:
+        if t.dtype != S.dtype or t.dim() != 2 or t.stride(1) != 1 or t.stride(0) != ld_T or not t.is_cuda:
+            raise ValueError("teacher buffers must be 2-D CUDA tensors of S's dtype with one row stride")
+    ptrs = (ctypes.c_void_p * D)(*[t.data_ptr() for t in T_domains])
+    nrows = (ctypes.c_int64 * D)(*[t.shape[0] for t in T_domains])
+    rows = int(row_end) - int(row_begin)
+    V = S.shape[1] if V is None else int(V)
+    n_traj = traj_row_off.numel() - 1
+    n_turns = turn_row_off.numel() - 1
+    lam_p, lam_all = _lambda(lam, n_traj)
+    rc = lib().stride_score_batch_multi_teacher(
+        S.data_ptr(), ptrs, nrows, D, ld_T, _dev(traj_domain, "traj_domain", torch.uint8, n_traj),
+        _dev(traj_T_row0, "traj_T_row0", torch.int64, n_traj), dt, S.stride(0), V,
+        _dev(tokens, "tokens", torch.int32, rows), _dev(traj_row_off, "traj_row_off", torch.int64),
+        _dev(turn_row_off, "turn_row_off", torch.int64), _dev(traj_turn_off, "traj_turn_off", torch.int32),
+        n_traj, n_turns, int(row_begin), int(row_end), int(stop_mode), lam_p, lam_all,
+        _dev(state, "state", torch.uint8, n_traj * STATE_DTYPE.itemsize), _row_outputs(out, rows),
+        _dev(turn_stats, "turn_stats", torch.uint8, n_turns * TURN_STATS_DTYPE.itemsize, optional=True),
+        _dev(profile, "profile", torch.float64, 3 * PROFILE_BINS, optional=True),
+        _dev(dev_status, "dev_status", torch.int32, 1, optional=True),
+        _dev(workspace, "workspace", torch.uint8, optional=True), 0 if workspace is None else workspace.numel(),
+        _stream(stream))
+    _check("stride_score_batch_multi_teacher", rc)
 
 
 def stride_buffer_record(buf_mean, buf_n_turns, task_of_traj, k0_of_traj, turn_stats, traj_turn_off,

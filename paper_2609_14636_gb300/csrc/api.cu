@@ -88,15 +88,21 @@ size_t stride_score_batch_workspace_size(int64_t window_rows) {
   return stride::batch_workspace_layout(window_rows).total;
 }
 
-int stride_score_batch(const void* S, const void* T, int32_t dtype, int64_t ld, int64_t V,
-                       const int32_t* tokens, const int64_t* traj_row_off,
-                       const int64_t* turn_row_off, const int32_t* traj_turn_off, int32_t n_traj,
-                       int32_t n_turns, int64_t row_begin, int64_t row_end, int32_t stop_mode,
-                       const float* lambda, float lambda_all, stride_scan_state* state,
-                       const stride_row_outputs* out, stride_turn_stats* turn_stats,
-                       double* profile, int32_t* dev_status, void* workspace,
-                       size_t workspace_bytes, void* stream) {
-  const int lc = check_logits(S, T, dtype, ld, V);
+}  // extern "C"
+
+namespace {
+
+// Checks and fills the parameters shared by the batch entry points; T may
+// be NULL when a teacher row table replaces it.
+int prepare_batch(stride::BatchParams& p, stride::BatchWorkspaceLayout& L, const void* S,
+                  const void* T, int32_t dtype, int64_t ld, int64_t V, const int32_t* tokens,
+                  const int64_t* traj_row_off, const int64_t* turn_row_off,
+                  const int32_t* traj_turn_off, int32_t n_traj, int32_t n_turns, int64_t row_begin,
+                  int64_t row_end, int32_t stop_mode, const float* lambda, float lambda_all,
+                  stride_scan_state* state, const stride_row_outputs* out,
+                  stride_turn_stats* turn_stats, double* profile, int32_t* dev_status,
+                  void* workspace, size_t workspace_bytes, size_t extra_ws_bytes) {
+  const int lc = check_logits(S, T ? T : S, dtype, ld, V);
   if (lc != STRIDE_OK) return lc;
   if (row_begin < 0 || row_end < row_begin || row_end - row_begin > INT32_MAX)
     return STRIDE_ERR_INVALID_ARG;
@@ -108,17 +114,17 @@ int stride_score_batch(const void* S, const void* T, int32_t dtype, int64_t ld, 
   const int64_t n_rows = row_end - row_begin;
   if (n_rows == 0) return STRIDE_OK;
   if (!tokens) return STRIDE_ERR_INVALID_ARG;
-  const stride::BatchWorkspaceLayout L = stride::batch_workspace_layout(n_rows);
-  if (!workspace || workspace_bytes < L.total ||
+  L = stride::batch_workspace_layout(n_rows);
+  if (!workspace || workspace_bytes < L.total + extra_ws_bytes ||
       (reinterpret_cast<uintptr_t>(workspace) & 255u) != 0)
     return STRIDE_ERR_WORKSPACE;
   const int dc = check_device();
   if (dc != STRIDE_OK) return dc;
-
   char* ws = static_cast<char*>(workspace);
-  stride::BatchParams p;
+  p = stride::BatchParams{};
   p.S = S;
   p.T = T;
+  p.T_rows = nullptr;
   p.ld = ld;
   p.V = (int32_t)V;
   p.mode = stop_mode;
@@ -142,11 +148,77 @@ int stride_score_batch(const void* S, const void* T, int32_t dtype, int64_t ld, 
   p.flags = reinterpret_cast<uint32_t*>(ws + L.flags_off);
   p.agg = reinterpret_cast<stride::ScanSlot*>(ws + L.agg_off);
   p.incl = reinterpret_cast<stride::ScanSlot*>(ws + L.incl_off);
-  p.timeout_ns = 2000000000ull;  // 2 s bound on any single lookback wait
+  p.timeout_ns = 2000000000ull;  // 2 s bound on any single device-side wait
+  return STRIDE_OK;
+}
 
+}  // namespace
+
+extern "C" {
+
+int stride_score_batch(const void* S, const void* T, int32_t dtype, int64_t ld, int64_t V,
+                       const int32_t* tokens, const int64_t* traj_row_off,
+                       const int64_t* turn_row_off, const int32_t* traj_turn_off, int32_t n_traj,
+                       int32_t n_turns, int64_t row_begin, int64_t row_end, int32_t stop_mode,
+                       const float* lambda, float lambda_all, stride_scan_state* state,
+                       const stride_row_outputs* out, stride_turn_stats* turn_stats,
+                       double* profile, int32_t* dev_status, void* workspace,
+                       size_t workspace_bytes, void* stream) {
+  if (!T) return STRIDE_ERR_INVALID_ARG;
+  stride::BatchParams p;
+  stride::BatchWorkspaceLayout L;
+  const int rc = prepare_batch(p, L, S, T, dtype, ld, V, tokens, traj_row_off, turn_row_off,
+                               traj_turn_off, n_traj, n_turns, row_begin, row_end, stop_mode, lambda,
+                               lambda_all, state, out, turn_stats, profile, dev_status, workspace,
+                               workspace_bytes, 0);
+  if (rc != STRIDE_OK || row_end == row_begin) return rc;
   cudaStream_t st = (cudaStream_t)stream;
-  if (cudaMemsetAsync(ws, 0, L.clear_bytes, st) != cudaSuccess) return STRIDE_ERR_CUDA;
+  if (cudaMemsetAsync(workspace, 0, L.clear_bytes, st) != cudaSuccess) return STRIDE_ERR_CUDA;
   const bool vec = vector_ok(S, T, dtype, ld);
+  return stride::launch_score_batch(p, dtype, vec, st) == cudaSuccess ? STRIDE_OK : STRIDE_ERR_CUDA;
+}
+
+int stride_score_batch_multi_teacher(const void* S, const void* const* T_domains,
+                                     const int64_t* T_domain_rows, int32_t n_domains, int64_t ld_T,
+                                     const uint8_t* traj_domain, const int64_t* traj_T_row0,
+                                     int32_t dtype, int64_t ld, int64_t V, const int32_t* tokens,
+                                     const int64_t* traj_row_off, const int64_t* turn_row_off,
+                                     const int32_t* traj_turn_off, int32_t n_traj, int32_t n_turns,
+                                     int64_t row_begin, int64_t row_end, int32_t stop_mode,
+                                     const float* lambda, float lambda_all, stride_scan_state* state,
+                                     const stride_row_outputs* out, stride_turn_stats* turn_stats,
+                                     double* profile, int32_t* dev_status, void* workspace,
+                                     size_t workspace_bytes, void* stream) {
+  if (!T_domains || !T_domain_rows || n_domains < 1 || n_domains > stride::kMaxTeacherDomains ||
+      !traj_domain || !traj_T_row0 || ld_T < V)
+    return STRIDE_ERR_INVALID_ARG;
+  stride::TeacherTable tt = {};
+  bool aligned = true;
+  for (int i = 0; i < n_domains; ++i) {
+    if (!T_domains[i] || T_domain_rows[i] < 0) return STRIDE_ERR_INVALID_ARG;
+    tt.base[i] = T_domains[i];
+    tt.rows[i] = T_domain_rows[i];
+    aligned = aligned && aligned16(T_domains[i]);
+  }
+  tt.n_domains = n_domains;
+  tt.ld_bytes = ld_T * (int64_t)dtype_bytes(dtype);
+  const int64_t n_rows = row_end > row_begin ? row_end - row_begin : 0;
+  const size_t table_bytes = ((size_t)n_rows * sizeof(void*) + 255) & ~size_t(255);
+  stride::BatchParams p;
+  stride::BatchWorkspaceLayout L;
+  const int rc = prepare_batch(p, L, S, nullptr, dtype, ld, V, tokens, traj_row_off, turn_row_off,
+                               traj_turn_off, n_traj, n_turns, row_begin, row_end, stop_mode, lambda,
+                               lambda_all, state, out, turn_stats, profile, dev_status, workspace,
+                               workspace_bytes, table_bytes);
+  if (rc != STRIDE_OK || n_rows == 0) return rc;
+  const void** rows = reinterpret_cast<const void**>(static_cast<char*>(workspace) + L.total);
+  cudaStream_t st = (cudaStream_t)stream;
+  if (cudaMemsetAsync(workspace, 0, L.clear_bytes, st) != cudaSuccess) return STRIDE_ERR_CUDA;
+  if (stride::launch_teacher_rows(p, tt, traj_domain, traj_T_row0, rows, st) != cudaSuccess)
+    return STRIDE_ERR_CUDA;
+  p.T_rows = rows;
+  const bool vec = aligned && aligned16(S) && ((ld * (int64_t)dtype_bytes(dtype)) % 16) == 0 &&
+                   (tt.ld_bytes % 16) == 0;
   return stride::launch_score_batch(p, dtype, vec, st) == cudaSuccess ? STRIDE_OK : STRIDE_ERR_CUDA;
 }
 

@@ -40,7 +40,7 @@ __global__ void __launch_bounds__(kBatchThreads, 2) score_batch_kernel(const Bat
   const int64_t tile = s_tile;
   const int64_t r = p.row_begin + tile;
   const LT* srow = reinterpret_cast<const LT*>(p.S) + tile * p.ld;
-  const LT* trow = reinterpret_cast<const LT*>(p.T) + tile * p.ld;
+  const LT* trow = teacher_row<LT>(p, tile);
 
   // Warp 0 starts the dependent lookups (token -> gathered logits, row ->
   // trajectory -> turn) before streaming, so their latency overlaps the
@@ -82,6 +82,39 @@ __global__ void __launch_bounds__(kBatchThreads, 2) score_batch_kernel(const Bat
   const float lse_t = lse_finish(mT, sT);
 
   finish_row(p, tile, r, meta, y, xs, xt, lse_s, lse_t, lane);
+}
+
+// Multi-teacher pre-pass: the teacher row of each window row, from its
+// trajectory's domain buffer.  A row whose domain or domain row is out of
+// range gets its domain-0 row 0 (always valid memory) and sets
+// STRIDE_DEV_BAD_LAYOUT: its results are meaningless, never a fault.
+__global__ void teacher_rows_kernel(const BatchParams p, const TeacherTable tt,
+                                    const uint8_t* __restrict__ traj_domain,
+                                    const int64_t* __restrict__ traj_T_row0, const void** rows_out) {
+  const int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (t >= p.n_rows) return;
+  const int64_t r = p.row_begin + t;
+  int64_t lo = 0, hi = p.n_traj - 1;  // largest i with traj_row_off[i] <= r
+  while (lo < hi) {
+    const int64_t mid = (lo + hi + 1) >> 1;
+    if (__ldg(p.traj_row_off + mid) <= r) lo = mid; else hi = mid - 1;
+  }
+  const int dom = __ldg(traj_domain + lo);
+  const int64_t tr = __ldg(traj_T_row0 + lo) + (r - __ldg(p.traj_row_off + lo));
+  const unsigned char* row = static_cast<const unsigned char*>(tt.base[0]);
+  if (dom < tt.n_domains && tr >= 0 && tr < tt.rows[dom] && r >= __ldg(p.traj_row_off)) {
+    row = static_cast<const unsigned char*>(tt.base[dom]) + tr * tt.ld_bytes;
+  } else {
+    set_status(p.dev_status, STRIDE_DEV_BAD_LAYOUT);
+  }
+  rows_out[t] = row;
+}
+
+cudaError_t launch_teacher_rows(const BatchParams& p, const TeacherTable& tt, const uint8_t* traj_domain,
+                                const int64_t* traj_T_row0, const void** rows_out, cudaStream_t stream) {
+  const unsigned grid = (unsigned)((p.n_rows + 255) / 256);
+  teacher_rows_kernel<<<grid, 256, 0, stream>>>(p, tt, traj_domain, traj_T_row0, rows_out);
+  return cudaGetLastError();
 }
 
 BatchWorkspaceLayout batch_workspace_layout(int64_t n_rows) {

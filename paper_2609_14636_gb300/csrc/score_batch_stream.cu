@@ -155,7 +155,7 @@ __global__ void __launch_bounds__(kStreamThreads, 1) score_batch_stream_kernel(c
         mbar_arrive(&sh.start[q]);
         if (done) break;
         const unsigned char* srow = reinterpret_cast<const unsigned char*>(p.S) + (int64_t)t * p.ld * sizeof(LT);
-        const unsigned char* trow = reinterpret_cast<const unsigned char*>(p.T) + (int64_t)t * p.ld * sizeof(LT);
+        const unsigned char* trow = reinterpret_cast<const unsigned char*>(teacher_row<LT>(p, (int64_t)t));
         for (int c = 0; c < n_chunks; ++c) {
           const int s = (int)(it % kStages);
           const uint32_t k = it / kStages;
@@ -301,7 +301,7 @@ __global__ void __launch_bounds__(kStreamThreads, 1) score_batch_stream_kernel(c
       }
       const int64_t r = p.row_begin + tile;
       const LT* srow = reinterpret_cast<const LT*>(p.S) + tile * p.ld;
-      const LT* trow = reinterpret_cast<const LT*>(p.T) + tile * p.ld;
+      const LT* trow = teacher_row<LT>(p, tile);
       int32_t y = 0;
       float xs = nan, xt = nan;
       if (lane == 0) {

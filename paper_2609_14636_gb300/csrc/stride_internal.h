@@ -19,6 +19,7 @@ struct alignas(32) ScanSlot {
 struct BatchParams {
   const void* S;
   const void* T;
+  const void* const* T_rows;  // per-window-row teacher row pointers (multi-teacher), or NULL
   int64_t ld;
   int32_t V;
   int32_t mode;
@@ -80,6 +81,24 @@ struct BatchWorkspaceLayout {
   size_t ticket_off, flags_off, agg_off, incl_off, clear_bytes, total;
 };
 BatchWorkspaceLayout batch_workspace_layout(int64_t n_rows);
+
+// Teacher row address of window row `tile`: the aligned T buffer, or the
+// multi-teacher row table.
+template <typename LT>
+__device__ __forceinline__ const LT* teacher_row(const BatchParams& p, int64_t tile) {
+  return p.T_rows ? reinterpret_cast<const LT*>(p.T_rows[tile])
+                  : reinterpret_cast<const LT*>(p.T) + tile * p.ld;
+}
+
+constexpr int kMaxTeacherDomains = 8;
+struct TeacherTable {
+  const void* base[kMaxTeacherDomains];
+  int64_t rows[kMaxTeacherDomains];
+  int32_t n_domains;
+  int64_t ld_bytes;
+};
+cudaError_t launch_teacher_rows(const BatchParams& p, const TeacherTable& tt, const uint8_t* traj_domain,
+                                const int64_t* traj_T_row0, const void** rows_out, cudaStream_t stream);
 
 // Launchers return a cudaError_t from the launch.
 cudaError_t launch_score_batch(const BatchParams& p, int dtype, bool vec, cudaStream_t stream);
