@@ -240,7 +240,7 @@ def load_lambda(w) -> np.ndarray:
     return np.full(w.layout.n_traj, np.float32(synth.workload_lambda(w.name)), np.float32)
 
 
-WORKLOADS = ("batch_scoring", "long_agentic", "multi_teacher", "decode_step", "select")
+WORKLOADS = ("batch_scoring", "long_agentic", "multi_teacher", "decode_step", "select", "tiny_reference")
 
 
 def main() -> None:
@@ -261,6 +261,8 @@ def main() -> None:
         return
     if args.workload == "decode_step":
         run_decode(args)
+    elif args.workload == "tiny_reference":
+        run_tiny(args)
     elif args.workload == "select":
         run_select(args)
     else:
@@ -624,6 +626,78 @@ def run_select(args) -> None:
                          "unit": "GB/s", "frac": None, "traffic": None, "us_per_call": us_call,
                          "kernel": "select_restart_kernel (one warp per record)"},
             "clocks": clk.summary(), "gpu_launches": reps * calls,
+        })
+        print(json.dumps(line), flush=True)
+
+
+def run_tiny(args) -> None:
+    """The tiny reference workload: 1 trajectory x 4 turns x 128 tokens,
+    V = 32,000 fp32 logits (131 MB, about the size of L2), token-sum stop
+    at lambda = -200.  L2 is flushed (a 512 MB write) before every timed
+    step; each step (state init + scoring) is timed with CUDA events."""
+    import torch
+
+    import oracle
+    import paper_2609_14636_gb300 as stride
+    import synth
+
+    ws, rank, local, dev = _setup_rank()
+    w = synth.tiny_reference(0)
+    lay = w["layout"]
+    R, V = lay.rows, w["V"]
+    S = torch.from_numpy(w["S"]).to(dev)
+    T = torch.from_numpy(w["T"]).to(dev)
+    tok = torch.from_numpy(w["tokens"]).to(dev)
+    offs = [torch.from_numpy(a).to(dev) for a in (lay.traj_row_off, lay.turn_row_off, lay.traj_turn_off)]
+    st = stride.new_state(lay.n_traj, dev)
+    ts = stride.new_turn_stats(lay.n_turns, dev)
+    out = {k: torch.empty(R, dtype=torch.float32, device=dev) for k in ("logp_s", "logp_t", "opd")}
+    status = torch.zeros(1, dtype=torch.int32, device=dev)
+    wsb = torch.empty(stride.stride_score_batch_workspace_size(R), dtype=torch.uint8, device=dev)
+    flush = torch.empty(512 << 20, dtype=torch.uint8, device=dev)
+    stream = torch.cuda.current_stream()
+
+    def step():
+        stride.stride_state_init(st, lay.n_traj, stream)
+        stride.stride_score_batch(S, T, tok, *offs, 0, R, stride.TOKEN_SUM, w["lam_token"], st, out=out,
+                                  turn_stats=ts, dev_status=status, workspace=wsb, stream=stream)
+
+    for _ in range(max(3, args.warmup)):
+        flush.zero_()
+        step()
+    torch.cuda.synchronize()
+    if int(status.item()) != 0:
+        raise RuntimeError(f"device status {int(status.item())}")
+    evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+    with ClockSampler(local) as clk:
+        time.sleep(0.25)
+        for a, b in evs:
+            flush.zero_()  # L2 flush, outside the timed events
+            a.record(stream)
+            step()
+            b.record(stream)
+        torch.cuda.synchronize()
+        time.sleep(0.05)
+    ms = statistics.mean(a.elapsed_time(b) for a, b in evs)
+    ms = max_over_ranks(ms, dev)
+    bpr = algorithmic_bytes_per_row(V, 4)
+    peak = measured_peaks().get("hbm_gbs", 6800.0)
+    threads = oracle.default_threads()
+    t0 = time.perf_counter()
+    oracle.row_logprobs(w["S"], w["T"], w["tokens"], nthreads=threads)
+    cpu_rate = R / (time.perf_counter() - t0)
+    if rank == 0:
+        line = _common_line(args, ws, ms, ws * R / (ms * 1e-3), dtype="f32")
+        line.update({
+            "config": {"workload": w["name"], "rows": R, "vocab": V, "stop_mode": "token_sum",
+                       "lambda": w["lam_token"], "l2": "512 MB written before every timed step (inputs 131 MB)"},
+            "roofline": {"bound": "hbm", "achieved": bpr * R / (ms * 1e-3) / 1e9, "peak": peak, "unit": "GB/s",
+                         "frac": bpr * R / (ms * 1e-3) / 1e9 / peak, "traffic": None,
+                         "algorithmic_bytes_per_launch": bpr * R, "kernel": "score_batch_stream_kernel<f32>",
+                         "note": "512 rows on 152 SMs: a latency-bound launch"},
+            "cpu_baseline": {"value": cpu_rate, "unit": UNIT, "cores": threads, "kind": "oracle",
+                             "sample": f"all {R} rows"},
+            "clocks": clk.summary(), "gpu_launches": 2 * args.steps,
         })
         print(json.dumps(line), flush=True)
 
