@@ -220,6 +220,46 @@ STRIDE_API int stride_score_batch_multi_teacher(
     stride_scan_state* state, const stride_row_outputs* out, stride_turn_stats* turn_stats,
     double* profile, int32_t* dev_status, void* workspace, size_t workspace_bytes, void* stream);
 
+/* ---- vocabulary-sharded logits and given log-probs -------------------------
+ * With tensor parallelism a model's logits are split by vocabulary columns
+ * across ranks.  Each rank reduces its shard (stride_partial_lse), the ranks
+ * exchange the 24-byte partials (all-gather; not done by this library), and
+ * stride_combine_partials forms the log-probs; stride_scan_logprobs then
+ * runs the rest of the path on them.  The result equals stride_score_batch
+ * on the full rows (Eq. 1, Eq. 4 log-softmax; the scan as in
+ * stride_score_batch). */
+
+/* Partial log-sum-exp of one vocabulary shard.  S, T: [rows, ld], this
+ * shard's V_shard columns (global columns col0 .. col0+V_shard-1); tokens:
+ * int32 [rows], global token ids.  partials: float [rows][6] =
+ * (m_S, s_S, m_T, s_T, S[y], T[y]) with LSE = m + ln(s) over the shard's
+ * columns, and the gathered logits NaN when y is not in this shard. */
+STRIDE_API int stride_partial_lse(const void* S, const void* T, int32_t dtype, int64_t ld,
+                                  int64_t V_shard, int64_t col0, const int32_t* tokens,
+                                  int64_t rows, float* partials, int32_t* dev_status, void* stream);
+
+/* Merges n_shards partials ([n_shards][rows][6], shard-major) into
+ * log-probs: LSE over all shards, the token's logit from the one shard that
+ * holds it (none or several: STRIDE_DEV_TOKEN_RANGE and NaN).  Outputs
+ * float [rows] each, nullable. */
+STRIDE_API int stride_combine_partials(const float* partials, int32_t n_shards, int64_t rows,
+                                       float* logp_s, float* logp_t, float* lse_s, float* lse_t,
+                                       int32_t* dev_status, void* stream);
+
+/* The scan part of stride_score_batch on given per-token log-probs
+ * (logp_s, logp_t: float, indexed by row - row_begin): d (opd, nullable),
+ * turn statistics, the stop rule, the OPD loss on retained tokens, the
+ * profile and the carried state, with the same layout, window, state and
+ * workspace rules (workspace: stride_score_batch_workspace_size(rows)). */
+STRIDE_API int stride_scan_logprobs(const float* logp_s, const float* logp_t,
+                                    const int64_t* traj_row_off, const int64_t* turn_row_off,
+                                    const int32_t* traj_turn_off, int32_t n_traj, int32_t n_turns,
+                                    int64_t row_begin, int64_t row_end, int32_t stop_mode,
+                                    const float* lambda, float lambda_all, stride_scan_state* state,
+                                    float* opd, stride_turn_stats* turn_stats, double* profile,
+                                    int32_t* dev_status, void* workspace, size_t workspace_bytes,
+                                    void* stream);
+
 /* One decode step over B rollouts (Algorithm 1, inner turn loop, one
  * generated token per rollout).
  *

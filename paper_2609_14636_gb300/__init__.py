@@ -30,7 +30,7 @@ __all__ = [
     "stride_select_restart", "stride_status_string", "stride_abi_version", "ROW_OUTPUT_KEYS",
     "stride_score_batch_noalloc", "NOALLOC_MAX_ROWS", "ERR_TOO_LARGE", "PROFILE_BINS", "new_profile",
     "stride_selftest_bounded_wait", "stride_buffer_record", "stride_score_batch_multi_teacher",
-    "multi_teacher_workspace_size",
+    "multi_teacher_workspace_size", "stride_partial_lse", "stride_combine_partials", "stride_scan_logprobs",
 ]
 
 DTYPE_BF16, DTYPE_F32 = 0, 1
@@ -82,6 +82,11 @@ def lib() -> ctypes.CDLL:
         L.stride_score_step.argtypes = [P, P, i32, i64, i64, P, P, i32, i32, P, f32, P, P, P, P, P, P]
         L.stride_select_restart.argtypes = [P, P, P, f32, i32, i32, P, P, P]
         L.stride_buffer_record.argtypes = [P, P, i32, i32, P, P, P, P, i32, P, P]
+        L.stride_partial_lse.argtypes = [P, P, i32, i64, i64, i64, P, i64, P, P, P]
+        L.stride_combine_partials.argtypes = [P, i32, i64, P, P, P, P, P, P]
+        L.stride_scan_logprobs.argtypes = [P, P, P, P, P, i32, i32, i64, i64, i32, P, f32, P, P, P, P, P, P, sz, P]
+        for fn in ("stride_partial_lse", "stride_combine_partials", "stride_scan_logprobs"):
+            getattr(L, fn).restype = ctypes.c_int
         L.stride_score_batch_multi_teacher.argtypes = [P, P, P, i32, i64, P, P, i32, i64, i64, P, P, P, P, i32,
                                                        i32, i64, i64, i32, P, f32, P, P, P, P, P, P, sz, P]
         L.stride_score_batch_multi_teacher.restype = ctypes.c_int
@@ -343,6 +348,60 @@ def stride_score_batch_multi_teacher(S, T_domains, traj_domain, traj_T_row0, tok
         _dev(workspace, "workspace", torch.uint8, optional=True), 0 if workspace is None else workspace.numel(),
         _stream(stream))
     _check("stride_score_batch_multi_teacher", rc)
+
+
+def stride_partial_lse(S, T, tokens, col0: int, partials, dev_status=None, V_shard: int | None = None,
+                       stream=None) -> None:
+    """Partial log-sum-exp of one vocabulary shard (columns col0 .. col0+V_shard-1
+    held in S, T [rows, ld]); partials: float32 [rows, 6]."""
+    torch = _torch()
+    dt, ld = _logits(S, T)
+    rows = S.shape[0]
+    V_shard = S.shape[1] if V_shard is None else int(V_shard)
+    rc = lib().stride_partial_lse(S.data_ptr(), T.data_ptr(), dt, ld, V_shard, int(col0),
+                                  _dev(tokens, "tokens", torch.int32, rows), rows,
+                                  _dev(partials, "partials", torch.float32, rows * 6),
+                                  _dev(dev_status, "dev_status", torch.int32, 1, optional=True), _stream(stream))
+    _check("stride_partial_lse", rc)
+
+
+def stride_combine_partials(partials, logp_s=None, logp_t=None, lse_s=None, lse_t=None, dev_status=None,
+                            stream=None) -> None:
+    """Merge float32 [n_shards, rows, 6] partials into log-probs."""
+    torch = _torch()
+    if partials.dim() != 3 or partials.shape[2] != 6:
+        raise ValueError("partials must be [n_shards, rows, 6]")
+    n, rows = partials.shape[0], partials.shape[1]
+    rc = lib().stride_combine_partials(
+        _dev(partials, "partials", torch.float32), n, rows, _dev(logp_s, "logp_s", torch.float32, rows, optional=True),
+        _dev(logp_t, "logp_t", torch.float32, rows, optional=True), _dev(lse_s, "lse_s", torch.float32, rows, optional=True),
+        _dev(lse_t, "lse_t", torch.float32, rows, optional=True),
+        _dev(dev_status, "dev_status", torch.int32, 1, optional=True), _stream(stream))
+    _check("stride_combine_partials", rc)
+
+
+def stride_scan_logprobs(logp_s, logp_t, traj_row_off, turn_row_off, traj_turn_off, row_begin: int, row_end: int,
+                         stop_mode: int, lam, state, opd=None, turn_stats=None, dev_status=None, workspace=None,
+                         stream=None, profile=None) -> None:
+    """The scan of stride_score_batch on given log-probs (float32, indexed by
+    row - row_begin)."""
+    torch = _torch()
+    rows = int(row_end) - int(row_begin)
+    n_traj = traj_row_off.numel() - 1
+    n_turns = turn_row_off.numel() - 1
+    lam_p, lam_all = _lambda(lam, n_traj)
+    rc = lib().stride_scan_logprobs(
+        _dev(logp_s, "logp_s", torch.float32, rows), _dev(logp_t, "logp_t", torch.float32, rows),
+        _dev(traj_row_off, "traj_row_off", torch.int64), _dev(turn_row_off, "turn_row_off", torch.int64),
+        _dev(traj_turn_off, "traj_turn_off", torch.int32), n_traj, n_turns, int(row_begin), int(row_end),
+        int(stop_mode), lam_p, lam_all, _dev(state, "state", torch.uint8, n_traj * STATE_DTYPE.itemsize),
+        _dev(opd, "opd", torch.float32, rows, optional=True),
+        _dev(turn_stats, "turn_stats", torch.uint8, n_turns * TURN_STATS_DTYPE.itemsize, optional=True),
+        _dev(profile, "profile", torch.float64, 3 * PROFILE_BINS, optional=True),
+        _dev(dev_status, "dev_status", torch.int32, 1, optional=True),
+        _dev(workspace, "workspace", torch.uint8, optional=True), 0 if workspace is None else workspace.numel(),
+        _stream(stream))
+    _check("stride_scan_logprobs", rc)
 
 
 def stride_buffer_record(buf_mean, buf_n_turns, task_of_traj, k0_of_traj, turn_stats, traj_turn_off,

@@ -281,6 +281,86 @@ int stride_select_restart(const float* turn_mean, const int32_t* n_turns, const 
                                                                               : STRIDE_ERR_CUDA;
 }
 
+int stride_partial_lse(const void* S, const void* T, int32_t dtype, int64_t ld, int64_t V_shard,
+                       int64_t col0, const int32_t* tokens, int64_t rows, float* partials,
+                       int32_t* dev_status, void* stream) {
+  const int lc = check_logits(S, T, dtype, ld, V_shard);
+  if (lc != STRIDE_OK) return lc;
+  if (rows < 0 || rows > INT32_MAX || col0 < 0) return STRIDE_ERR_INVALID_ARG;
+  if (rows == 0) return STRIDE_OK;
+  if (!tokens || !partials) return STRIDE_ERR_INVALID_ARG;
+  const int dc = check_device();
+  if (dc != STRIDE_OK) return dc;
+  return stride::launch_partial_lse(S, T, dtype, vector_ok(S, T, dtype, ld), ld, (int32_t)V_shard, col0,
+                                    tokens, rows, partials, dev_status, (cudaStream_t)stream) == cudaSuccess
+             ? STRIDE_OK
+             : STRIDE_ERR_CUDA;
+}
+
+int stride_combine_partials(const float* partials, int32_t n_shards, int64_t rows, float* logp_s,
+                            float* logp_t, float* lse_s, float* lse_t, int32_t* dev_status,
+                            void* stream) {
+  if (n_shards < 1 || rows < 0) return STRIDE_ERR_INVALID_ARG;
+  if (rows == 0) return STRIDE_OK;
+  if (!partials) return STRIDE_ERR_INVALID_ARG;
+  const int dc = check_device();
+  if (dc != STRIDE_OK) return dc;
+  return stride::launch_combine_partials(partials, n_shards, rows, logp_s, logp_t, lse_s, lse_t, dev_status,
+                                         (cudaStream_t)stream) == cudaSuccess
+             ? STRIDE_OK
+             : STRIDE_ERR_CUDA;
+}
+
+int stride_scan_logprobs(const float* logp_s, const float* logp_t, const int64_t* traj_row_off,
+                         const int64_t* turn_row_off, const int32_t* traj_turn_off, int32_t n_traj,
+                         int32_t n_turns, int64_t row_begin, int64_t row_end, int32_t stop_mode,
+                         const float* lambda, float lambda_all, stride_scan_state* state, float* opd,
+                         stride_turn_stats* turn_stats, double* profile, int32_t* dev_status,
+                         void* workspace, size_t workspace_bytes, void* stream) {
+  if (row_begin < 0 || row_end < row_begin || row_end - row_begin > INT32_MAX)
+    return STRIDE_ERR_INVALID_ARG;
+  if (stop_mode != STRIDE_STOP_TURN_MEAN && stop_mode != STRIDE_STOP_TOKEN_SUM)
+    return STRIDE_ERR_INVALID_ARG;
+  if (n_traj < 1 || n_turns < 0 || !traj_row_off || !turn_row_off || !traj_turn_off || !state)
+    return STRIDE_ERR_INVALID_ARG;
+  if (!lambda && isnan(lambda_all)) return STRIDE_ERR_INVALID_ARG;
+  const int64_t n_rows = row_end - row_begin;
+  if (n_rows == 0) return STRIDE_OK;
+  if (!logp_s || !logp_t) return STRIDE_ERR_INVALID_ARG;
+  const stride::BatchWorkspaceLayout L = stride::batch_workspace_layout(n_rows);
+  if (!workspace || workspace_bytes < L.total || (reinterpret_cast<uintptr_t>(workspace) & 255u) != 0)
+    return STRIDE_ERR_WORKSPACE;
+  const int dc = check_device();
+  if (dc != STRIDE_OK) return dc;
+  char* ws = static_cast<char*>(workspace);
+  stride::BatchParams p = {};
+  p.V = 1;
+  p.mode = stop_mode;
+  p.traj_row_off = traj_row_off;
+  p.turn_row_off = turn_row_off;
+  p.traj_turn_off = traj_turn_off;
+  p.n_traj = n_traj;
+  p.n_turns = n_turns;
+  p.row_begin = row_begin;
+  p.row_end = row_end;
+  p.n_rows = n_rows;
+  p.lambda = lambda;
+  p.lambda_all = lambda_all;
+  p.state = state;
+  p.out = stride_row_outputs{nullptr, nullptr, opd, nullptr, nullptr, nullptr, nullptr};
+  p.turn_stats = turn_stats;
+  p.profile = profile;
+  p.dev_status = dev_status;
+  p.ticket = reinterpret_cast<uint32_t*>(ws + L.ticket_off);
+  p.flags = reinterpret_cast<uint32_t*>(ws + L.flags_off);
+  p.agg = reinterpret_cast<stride::ScanSlot*>(ws + L.agg_off);
+  p.incl = reinterpret_cast<stride::ScanSlot*>(ws + L.incl_off);
+  p.timeout_ns = 2000000000ull;
+  cudaStream_t st = (cudaStream_t)stream;
+  if (cudaMemsetAsync(workspace, 0, L.clear_bytes, st) != cudaSuccess) return STRIDE_ERR_CUDA;
+  return stride::launch_scan_logprobs(p, logp_s, logp_t, st) == cudaSuccess ? STRIDE_OK : STRIDE_ERR_CUDA;
+}
+
 int stride_buffer_record(float* buf_mean, int32_t* buf_n_turns, int32_t n_tasks, int32_t T_max,
                          const int32_t* task_of_traj, const int32_t* k0_of_traj,
                          const stride_turn_stats* turn_stats, const int32_t* traj_turn_off,

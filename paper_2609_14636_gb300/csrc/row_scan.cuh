@@ -231,7 +231,7 @@ struct RowCarry {
 };
 
 __device__ __forceinline__ RowCarry row_finalize(const BatchParams& p, int64_t tile, int64_t r,
-                                                 const RowMeta& meta, int32_t y, float xs, float xt,
+                                                 const RowMeta& meta, bool token_ok, float xs, float xt,
                                                  float lse_s, float lse_t, double* prof,
                                                  bool prof_atomic) {
   RowCarry rc;
@@ -239,7 +239,7 @@ __device__ __forceinline__ RowCarry row_finalize(const BatchParams& p, int64_t t
   const float nan = __int_as_float(0x7fc00000);
   float lps = xs - lse_s;
   float lpt = xt - lse_t;
-  if (!(y >= 0 && y < p.V)) set_status(p.dev_status, STRIDE_DEV_TOKEN_RANGE);
+  if (!token_ok) set_status(p.dev_status, STRIDE_DEV_TOKEN_RANGE);
   if (meta.bad) {
     set_status(p.dev_status, STRIDE_DEV_BAD_LAYOUT);
     lps = nan;
@@ -375,7 +375,7 @@ __device__ __forceinline__ void finish_row(const BatchParams& p, int64_t tile, i
                                            const RowMeta& meta, int32_t y, float xs, float xt,
                                            float lse_s, float lse_t, int lane) {
   RowCarry rc;
-  if (lane == 0) rc = row_finalize(p, tile, r, meta, y, xs, xt, lse_s, lse_t, p.profile, true);
+  if (lane == 0) rc = row_finalize(p, tile, r, meta, y >= 0 && y < p.V, xs, xt, lse_s, lse_t, p.profile, true);
   row_resolve(p, tile, r, meta, rc, lane);
 }
 

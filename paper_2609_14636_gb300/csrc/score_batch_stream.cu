@@ -329,8 +329,8 @@ __global__ void __launch_bounds__(kStreamThreads, 1) score_batch_stream_kernel(c
       lse_merge(mS, sS, tmS, tsS);
       lse_merge(mT, sT, tmT, tsT);
       if (lane == 0) {
-        sh.slot_carry[q] = row_finalize(p, tile, r, meta, y, xs, xt, lse_finish(mS, sS), lse_finish(mT, sT),
-                                        p.profile ? sh.prof : nullptr, false);
+        sh.slot_carry[q] = row_finalize(p, tile, r, meta, y >= 0 && y < p.V, xs, xt, lse_finish(mS, sS),
+                                        lse_finish(mT, sT), p.profile ? sh.prof : nullptr, false);
         sh.slot_meta[q] = meta;
         mbar_arrive(&sh.agg_ready[q]);
       }

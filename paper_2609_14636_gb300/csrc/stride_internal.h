@@ -106,6 +106,14 @@ cudaError_t launch_score_batch_stream(const BatchParams& p, int dtype, cudaStrea
 cudaError_t launch_score_step(const StepParams& p, int dtype, bool vec, cudaStream_t stream);
 cudaError_t launch_select_restart(const SelectParams& p, cudaStream_t stream);
 cudaError_t launch_state_init(stride_scan_state* state, int32_t n, cudaStream_t stream);
+cudaError_t launch_partial_lse(const void* S, const void* T, int dtype, bool vec, int64_t ld,
+                               int32_t V_shard, int64_t col0, const int32_t* tokens, int64_t rows,
+                               float* partials, int32_t* dev_status, cudaStream_t stream);
+cudaError_t launch_combine_partials(const float* parts, int32_t n_shards, int64_t rows, float* logp_s,
+                                    float* logp_t, float* lse_s, float* lse_t, int32_t* dev_status,
+                                    cudaStream_t stream);
+cudaError_t launch_scan_logprobs(const BatchParams& p, const float* logp_s, const float* logp_t,
+                                 cudaStream_t stream);
 cudaError_t launch_buffer_record(float* buf_mean, int32_t* buf_n_turns, int32_t n_tasks, int32_t T_max,
                                  const int32_t* task, const int32_t* k0, const stride_turn_stats* ts,
                                  const int32_t* traj_turn_off, int32_t n_traj, int32_t* dev_status,
