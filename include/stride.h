@@ -50,6 +50,12 @@
  *   in a CUDA graph.
  * - The library is built for sm_103a only; on another device the calls return
  *   STRIDE_ERR_UNSUPPORTED_DEVICE.  There is no CPU fallback.
+ * - The batch calls choose among three kernels with the same results: a
+ *   4-CTA-cluster kernel for windows of fewer than 8 rows per SM, a
+ *   persistent bulk-copy kernel for 16-byte-aligned rows, and one CTA per
+ *   row otherwise.  The environment variable STRIDE_BATCH_KERNEL=split,
+ *   stream or rows forces one of them (for tests and diagnosis; stream
+ *   still needs aligned rows, split needs V >= 128).
  */
 #ifndef STRIDE_H_
 #define STRIDE_H_

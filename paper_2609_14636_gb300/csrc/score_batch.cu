@@ -15,7 +15,10 @@
 //      lambda with atomicMin (Eq. 5 / Sec. 5.5).
 //
 // The row tail (steps 2-4) and the scan protocol live in row_scan.cuh.
+#include <cooperative_groups.h>
 #include <math.h>
+#include <stdlib.h>
+#include <string.h>
 
 #include "stride.h"
 #include "stride_device.cuh"
@@ -84,6 +87,103 @@ __global__ void __launch_bounds__(kBatchThreads, 2) score_batch_kernel(const Bat
   finish_row(p, tile, r, meta, y, xs, xt, lse_s, lse_t, lane);
 }
 
+// Small windows: a few rows per SM leave the persistent kernel latency-bound
+// (each SM streams its rows one after another), so a window of fewer than
+// kSplitRowsPerSm rows per SM splits every row over the kSplitCluster CTAs of
+// a thread-block cluster instead.  Rank 0 takes the row's ticket and shares
+// it through distributed shared memory; every rank streams its share of the
+// vocabulary of S and T; rank 0 merges the ranks' pairs, then runs the row
+// tail (finalize, lookback, resolve) after the other ranks have left.
+namespace cg = cooperative_groups;
+constexpr int kSplitCluster = 4;
+constexpr int kSplitThreads = 128;
+constexpr int kSplitWarps = kSplitThreads / 32;
+
+template <typename LT, bool VEC>
+__global__ void __cluster_dims__(kSplitCluster, 1, 1) __launch_bounds__(kSplitThreads, 8)
+    score_batch_split_kernel(const BatchParams p) {
+  __shared__ float s_red[4][kSplitWarps];
+  __shared__ float s_part[4];
+  __shared__ int64_t s_tile;
+  cg::cluster_group cluster = cg::this_cluster();
+  const int rank = (int)cluster.block_rank();
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  if (rank == 0 && tid == 0) s_tile = (int64_t)atomicAdd(p.ticket, 1u);
+  cluster.sync();
+  const int64_t tile = *cluster.map_shared_rank(&s_tile, 0);
+  const int64_t r = p.row_begin + tile;
+  const LT* srow = reinterpret_cast<const LT*>(p.S) + tile * p.ld;
+  const LT* trow = teacher_row<LT>(p, tile);
+
+  int32_t y = 0;
+  float xs = __int_as_float(0x7fc00000), xt = xs;
+  RowMeta meta;
+  if (rank == 0 && warp == 0) {
+    if (lane == 0) {
+      y = __ldg(p.tokens + tile);
+      if (y >= 0 && y < p.V) {
+        xs = to_f32(srow[y]);
+        xt = to_f32(trow[y]);
+      }
+      validate_layout(p, tile);
+    }
+    meta = find_row_meta(p, r, lane);
+  }
+  int c0, c1;
+  if (VEC) {
+    constexpr int P = LogitTraits<LT>::kPerVec;
+    const int nv = p.V / P;
+    const int per = (nv + kSplitCluster - 1) / kSplitCluster;
+    c0 = min(nv, rank * per) * P;
+    c1 = (rank == kSplitCluster - 1) ? p.V : min(nv, (rank + 1) * per) * P;
+  } else {
+    const int per = (p.V + kSplitCluster - 1) / kSplitCluster;
+    c0 = min(p.V, rank * per);
+    c1 = min(p.V, (rank + 1) * per);
+  }
+  float mS = kMaxStart, sS = 0.f, mT = kMaxStart, sT = 0.f;
+  stream_pair<LT, VEC, 4>(srow, trow, c0, c1, tid, kSplitThreads, mS, sS, mT, sT);
+  warp_merge2(mS, sS, mT, sT);
+  if (lane == 0) {
+    s_red[0][warp] = mS;
+    s_red[1][warp] = sS;
+    s_red[2][warp] = mT;
+    s_red[3][warp] = sT;
+  }
+  __syncthreads();
+  if (warp == 0) {
+    mS = lane < kSplitWarps ? s_red[0][lane] : kMaxStart;
+    sS = lane < kSplitWarps ? s_red[1][lane] : 0.f;
+    mT = lane < kSplitWarps ? s_red[2][lane] : kMaxStart;
+    sT = lane < kSplitWarps ? s_red[3][lane] : 0.f;
+    warp_merge2(mS, sS, mT, sT);
+    if (lane == 0) {
+      s_part[0] = mS;
+      s_part[1] = sS;
+      s_part[2] = mT;
+      s_part[3] = sT;
+    }
+  }
+  cluster.sync();
+  if (rank == 0 && warp == 0) {
+    mS = kMaxStart;
+    sS = 0.f;
+    mT = kMaxStart;
+    sT = 0.f;
+    if (lane < kSplitCluster) {
+      const float* peer = cluster.map_shared_rank(s_part, lane);
+      mS = peer[0];
+      sS = peer[1];
+      mT = peer[2];
+      sT = peer[3];
+    }
+    warp_merge2(mS, sS, mT, sT);
+  }
+  cluster.sync();  // the ranks' shared memory has been read: they may leave
+  if (rank != 0 || warp != 0) return;
+  finish_row(p, tile, r, meta, y, xs, xt, lse_finish(mS, sS), lse_finish(mT, sT), lane);
+}
+
 // Multi-teacher pre-pass: the teacher row of each window row, from its
 // trajectory's domain buffer.  A row whose domain or domain row is out of
 // range gets its domain-0 row 0 (always valid memory) and sets
@@ -131,11 +231,44 @@ BatchWorkspaceLayout batch_workspace_layout(int64_t n_rows) {
   return L;
 }
 
+#ifndef STRIDE_SPLIT_ROWS_PER_SM
+#define STRIDE_SPLIT_ROWS_PER_SM 8
+#endif
+
 cudaError_t launch_score_batch(const BatchParams& p, int dtype, bool vec, cudaStream_t stream) {
-  // 16-byte-aligned rows with at least one whole vector take the persistent
-  // bulk-copy kernel (score_batch_stream.cu); the rest take one CTA per row.
+  // Windows of fewer than STRIDE_SPLIT_ROWS_PER_SM rows per SM split each
+  // row over a 4-CTA cluster; 16-byte-aligned rows with at least one whole
+  // vector otherwise take the persistent bulk-copy kernel
+  // (score_batch_stream.cu); the rest take one CTA per row.
+  static int sm_count[64] = {0};
+  int dev = 0;
+  if (cudaGetDevice(&dev) == cudaSuccess && dev >= 0 && dev < 64 && sm_count[dev] == 0)
+    cudaDeviceGetAttribute(&sm_count[dev], cudaDevAttrMultiProcessorCount, dev);
+  const int sms = (dev >= 0 && dev < 64 && sm_count[dev] > 0) ? sm_count[dev] : 152;
+  // STRIDE_BATCH_KERNEL = split | stream | rows forces one kernel (tests and
+  // diagnosis); anything else, or unset, chooses by window size.
+  const char* force = getenv("STRIDE_BATCH_KERNEL");
+  const bool f_split = force && !strcmp(force, "split");
+  const bool f_stream = force && !strcmp(force, "stream");
+  const bool f_rows = force && !strcmp(force, "rows");
+  const bool split_ok = p.V >= 4 * kSplitCluster * 8;
+  if (split_ok && (f_split || (!f_stream && !f_rows && p.n_rows < (int64_t)STRIDE_SPLIT_ROWS_PER_SM * sms))) {
+    const dim3 grid((unsigned)(p.n_rows * kSplitCluster)), block(kSplitThreads);
+    if (dtype == STRIDE_DTYPE_BF16) {
+      if (vec)
+        score_batch_split_kernel<__nv_bfloat16, true><<<grid, block, 0, stream>>>(p);
+      else
+        score_batch_split_kernel<__nv_bfloat16, false><<<grid, block, 0, stream>>>(p);
+    } else {
+      if (vec)
+        score_batch_split_kernel<float, true><<<grid, block, 0, stream>>>(p);
+      else
+        score_batch_split_kernel<float, false><<<grid, block, 0, stream>>>(p);
+    }
+    return cudaGetLastError();
+  }
   const int per_vec = dtype == STRIDE_DTYPE_BF16 ? 8 : 4;
-  if (vec && p.V >= per_vec) return launch_score_batch_stream(p, dtype, stream);
+  if (vec && p.V >= per_vec && !f_rows) return launch_score_batch_stream(p, dtype, stream);
   const dim3 grid((unsigned)p.n_rows), block(kBatchThreads);
   if (dtype == STRIDE_DTYPE_BF16) {
     if (vec)

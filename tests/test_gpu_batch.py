@@ -22,6 +22,17 @@ def stride():
     return s
 
 
+@pytest.fixture(params=["auto", "stream", "split", "rows"])
+def kernel(request, monkeypatch):
+    """Runs a test under each of the batch kernels (the library reads
+    STRIDE_BATCH_KERNEL on every call)."""
+    if request.param == "auto":
+        monkeypatch.delenv("STRIDE_BATCH_KERNEL", raising=False)
+    else:
+        monkeypatch.setenv("STRIDE_BATCH_KERNEL", request.param)
+    return request.param
+
+
 def _bf16_rows(seed, R, V, sigma=4.0, noise=0.5):
     rng = np.random.default_rng(seed)
     S32 = (rng.standard_normal((R, V), dtype=np.float32) * np.float32(sigma))
@@ -52,7 +63,7 @@ def _lam_between_turns(o, lay, targets):
 # tiny reference workload: 1 x 4 turns x 128 tokens, V = 32,000, fp32
 # ---------------------------------------------------------------------------
 @pytest.mark.parametrize("mode,lam_key", [(1, "lam_token"), (0, "lam_turn")])
-def test_tiny_reference(stride, mode, lam_key):
+def test_tiny_reference(stride, kernel, mode, lam_key):
     w = synth.tiny_reference(0)
     g = run_batch(stride, w["S"], w["T"], w["tokens"], w["layout"], mode, w[lam_key])
     o = oracle_batch(w["S"], w["T"], w["tokens"], w["layout"], mode, w[lam_key])
@@ -71,7 +82,7 @@ LENS = [[1, 5, 17, 3], [9, 1], [33, 2, 1, 1, 4], [2]]
 @pytest.mark.parametrize("V,ld", [(151_936, 151_936), (151_933, 151_936), (151_933, 151_933),
                                   (4099, 4099), (8, 8), (7, 8), (1, 1), (1, 8)])
 @pytest.mark.parametrize("mode", [0, 1])
-def test_bf16_ragged(stride, V, ld, mode):
+def test_bf16_ragged(stride, kernel, V, ld, mode):
     lay = synth.layout_from_turn_lengths(LENS)
     S, T, tok = _bf16_rows(V + ld, lay.rows, V)
     Sp, Tp = pad_cols(S, ld, 0x7FC0), pad_cols(T, ld, 0x7FC0)  # NaN padding must never be read
@@ -88,7 +99,7 @@ def test_bf16_ragged(stride, V, ld, mode):
     compare_scan(g, o, lay, mode, lam)
 
 
-def test_f32_vector_and_scalar_paths(stride):
+def test_f32_vector_and_scalar_paths(stride, kernel):
     rng = np.random.default_rng(5)
     lay = synth.layout_from_turn_lengths([[7, 3], [11]])
     V = 32_000
@@ -107,7 +118,7 @@ def test_f32_vector_and_scalar_paths(stride):
 # chunked windows: same results as one call and as the oracle
 # ---------------------------------------------------------------------------
 @pytest.mark.parametrize("mode", [0, 1])
-def test_chunked_windows(stride, mode):
+def test_chunked_windows(stride, kernel, mode):
     rng = np.random.default_rng(9)
     lay = synth.ragged_layout(rng, 6, (1, 7), 1, 60)
     V = 3000
@@ -132,7 +143,7 @@ def test_chunked_windows(stride, mode):
         assert np.array_equal(g["turn_stats"]["n"], one["turn_stats"]["n"])
 
 
-def test_many_tiles(stride):
+def test_many_tiles(stride, kernel):
     """Thousands of tiles, hundreds of trajectories, single-row turns: the
     lookback chain crosses many trajectory and turn boundaries."""
     rng = np.random.default_rng(21)
@@ -184,7 +195,7 @@ def test_identical_rows_zero_opd(stride):
     assert np.array_equal(g["turn_stats"]["sum_d"], np.zeros(2))
 
 
-def test_masked_vocab_entries(stride):
+def test_masked_vocab_entries(stride, kernel):
     """-inf logits carry no probability mass."""
     lay = synth.layout_from_turn_lengths([[6]])
     V = 5000
@@ -199,7 +210,7 @@ def test_masked_vocab_entries(stride):
     assert g["logp_s"][3] == -np.inf
 
 
-def test_token_out_of_range_sets_status(stride):
+def test_token_out_of_range_sets_status(stride, kernel):
     lay = synth.layout_from_turn_lengths([[4], [3]])
     S, T, tok = _bf16_rows(51, lay.rows, 1000)
     tok[1] = 1000
