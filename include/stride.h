@@ -50,12 +50,14 @@
  *   in a CUDA graph.
  * - The library is built for sm_103a only; on another device the calls return
  *   STRIDE_ERR_UNSUPPORTED_DEVICE.  There is no CPU fallback.
- * - The batch calls choose among three kernels with the same results: a
- *   4-CTA-cluster kernel for windows of fewer than 8 rows per SM, a
- *   persistent bulk-copy kernel for 16-byte-aligned rows, and one CTA per
+ * - The batch calls choose among three kernels with the same results: for
+ *   windows of at most 8 rows per SM, a kernel that splits each row over a
+ *   thread-block cluster of 1, 2, 4 or 8 CTAs (the window is one wave); a
+ *   persistent bulk-copy kernel for 16-byte-aligned rows; and one CTA per
  *   row otherwise.  The environment variable STRIDE_BATCH_KERNEL=split,
- *   stream or rows forces one of them (for tests and diagnosis; stream
- *   still needs aligned rows, split needs V >= 128).
+ *   stream or rows forces one of them, split1, split2, split4 or split8 the
+ *   split kernel with that cluster size (for tests and diagnosis; stream
+ *   still needs aligned rows).
  */
 #ifndef STRIDE_H_
 #define STRIDE_H_

@@ -88,25 +88,29 @@ __global__ void __launch_bounds__(kBatchThreads, 2) score_batch_kernel(const Bat
 }
 
 // Small windows: a few rows per SM leave the persistent kernel latency-bound
-// (each SM streams its rows one after another), so a window of fewer than
-// kSplitRowsPerSm rows per SM splits every row over the kSplitCluster CTAs of
-// a thread-block cluster instead.  Rank 0 takes the row's ticket and shares
-// it through distributed shared memory; every rank streams its share of the
-// vocabulary of S and T; rank 0 merges the ranks' pairs, then runs the row
-// tail (finalize, lookback, resolve) after the other ranks have left.
+// (each SM streams its rows one after another), so a window of at most 8
+// rows per SM splits every row over the C CTAs of a thread-block cluster
+// instead (C = 1: one CTA per row), C chosen at launch (split_cluster below)
+// so that the window is one wave of 128-thread CTAs.  Rank 0 takes the row's
+// ticket and shares it through distributed shared memory; every rank streams
+// its share of the vocabulary of S and T; rank 0 merges the ranks' pairs,
+// then runs the row tail (finalize, lookback, resolve) after the other ranks
+// have left.
 namespace cg = cooperative_groups;
-constexpr int kSplitCluster = 4;
+constexpr int kSplitMaxCluster = 8;
 constexpr int kSplitThreads = 128;
 constexpr int kSplitWarps = kSplitThreads / 32;
+constexpr int kSplitBlocksPerSm = 8;  // 128 threads at <= 64 registers
 
 template <typename LT, bool VEC>
-__global__ void __cluster_dims__(kSplitCluster, 1, 1) __launch_bounds__(kSplitThreads, 8)
+__global__ void __launch_bounds__(kSplitThreads, kSplitBlocksPerSm)
     score_batch_split_kernel(const BatchParams p) {
   __shared__ float s_red[4][kSplitWarps];
   __shared__ float s_part[4];
   __shared__ int64_t s_tile;
   cg::cluster_group cluster = cg::this_cluster();
   const int rank = (int)cluster.block_rank();
+  const int n_ranks = (int)cluster.num_blocks();
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   if (rank == 0 && tid == 0) s_tile = (int64_t)atomicAdd(p.ticket, 1u);
   cluster.sync();
@@ -133,11 +137,11 @@ __global__ void __cluster_dims__(kSplitCluster, 1, 1) __launch_bounds__(kSplitTh
   if (VEC) {
     constexpr int P = LogitTraits<LT>::kPerVec;
     const int nv = p.V / P;
-    const int per = (nv + kSplitCluster - 1) / kSplitCluster;
+    const int per = (nv + n_ranks - 1) / n_ranks;
     c0 = min(nv, rank * per) * P;
-    c1 = (rank == kSplitCluster - 1) ? p.V : min(nv, (rank + 1) * per) * P;
+    c1 = (rank == n_ranks - 1) ? p.V : min(nv, (rank + 1) * per) * P;
   } else {
-    const int per = (p.V + kSplitCluster - 1) / kSplitCluster;
+    const int per = (p.V + n_ranks - 1) / n_ranks;
     c0 = min(p.V, rank * per);
     c1 = min(p.V, (rank + 1) * per);
   }
@@ -170,7 +174,7 @@ __global__ void __cluster_dims__(kSplitCluster, 1, 1) __launch_bounds__(kSplitTh
     sS = 0.f;
     mT = kMaxStart;
     sT = 0.f;
-    if (lane < kSplitCluster) {
+    if (lane < n_ranks) {
       const float* peer = cluster.map_shared_rank(s_part, lane);
       mS = peer[0];
       sS = peer[1];
@@ -231,40 +235,75 @@ BatchWorkspaceLayout batch_workspace_layout(int64_t n_rows) {
   return L;
 }
 
-#ifndef STRIDE_SPLIT_ROWS_PER_SM
-#define STRIDE_SPLIT_ROWS_PER_SM 8
+// Cluster size of the small-window kernel: the largest C in {8, 4, 2, 1}
+// whose n_rows * C CTAs fit in one wave (kSplitBlocksPerSm per SM), 0 when
+// even C = 1 does not (the window then takes the persistent kernel).  A
+// sweep on GB300 over windows of 64..2,432 rows (bf16 V = 151,936 and fp32
+// V = 32,000) found this choice within a few percent of the best cluster size
+// at every window, and up to 1,216 rows faster than the persistent kernel,
+// which streams each SM's few rows one after another; from 1,600 rows on the
+// persistent kernel is faster.
+// STRIDE_SPLIT_FORCE_CLUSTER (a build define) fixes C for launch-shape sweeps.
+#ifndef STRIDE_SPLIT_FORCE_CLUSTER
+#define STRIDE_SPLIT_FORCE_CLUSTER 0
 #endif
+static int split_cluster(int64_t n_rows, int sms) {
+  if (STRIDE_SPLIT_FORCE_CLUSTER > 0) return STRIDE_SPLIT_FORCE_CLUSTER;
+  const int64_t slots = (int64_t)kSplitBlocksPerSm * sms;
+  for (int c = kSplitMaxCluster; c >= 1; c >>= 1)
+    if (n_rows * c <= slots) return c;
+  return 0;
+}
+
+template <typename LT, bool VEC>
+static cudaError_t launch_split(const BatchParams& p, int C, cudaStream_t stream) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)(p.n_rows * C));
+  cfg.blockDim = dim3(kSplitThreads);
+  cfg.dynamicSmemBytes = 0;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = (unsigned)C;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, score_batch_split_kernel<LT, VEC>, p);
+}
 
 cudaError_t launch_score_batch(const BatchParams& p, int dtype, bool vec, cudaStream_t stream) {
-  // Windows of fewer than STRIDE_SPLIT_ROWS_PER_SM rows per SM split each
-  // row over a 4-CTA cluster; 16-byte-aligned rows with at least one whole
-  // vector otherwise take the persistent bulk-copy kernel
-  // (score_batch_stream.cu); the rest take one CTA per row.
+  // Small windows split each row over a cluster (split_cluster); 16-byte-
+  // aligned rows with at least one whole vector otherwise take the
+  // persistent bulk-copy kernel (score_batch_stream.cu); the rest take one
+  // CTA per row.
   static int sm_count[64] = {0};
   int dev = 0;
   if (cudaGetDevice(&dev) == cudaSuccess && dev >= 0 && dev < 64 && sm_count[dev] == 0)
     cudaDeviceGetAttribute(&sm_count[dev], cudaDevAttrMultiProcessorCount, dev);
   const int sms = (dev >= 0 && dev < 64 && sm_count[dev] > 0) ? sm_count[dev] : 152;
-  // STRIDE_BATCH_KERNEL = split | stream | rows forces one kernel (tests and
-  // diagnosis); anything else, or unset, chooses by window size.
+  // STRIDE_BATCH_KERNEL = split | split1 | split2 | split4 | split8 |
+  // stream | rows forces one kernel, or the split kernel with one cluster
+  // size (tests and diagnosis); anything else, or unset, chooses by window
+  // size.
   const char* force = getenv("STRIDE_BATCH_KERNEL");
-  const bool f_split = force && !strcmp(force, "split");
+  const bool f_split = force && !strncmp(force, "split", 5);
   const bool f_stream = force && !strcmp(force, "stream");
   const bool f_rows = force && !strcmp(force, "rows");
-  const bool split_ok = p.V >= 4 * kSplitCluster * 8;
-  if (split_ok && (f_split || (!f_stream && !f_rows && p.n_rows < (int64_t)STRIDE_SPLIT_ROWS_PER_SM * sms))) {
-    const dim3 grid((unsigned)(p.n_rows * kSplitCluster)), block(kSplitThreads);
-    if (dtype == STRIDE_DTYPE_BF16) {
-      if (vec)
-        score_batch_split_kernel<__nv_bfloat16, true><<<grid, block, 0, stream>>>(p);
-      else
-        score_batch_split_kernel<__nv_bfloat16, false><<<grid, block, 0, stream>>>(p);
-    } else {
-      if (vec)
-        score_batch_split_kernel<float, true><<<grid, block, 0, stream>>>(p);
-      else
-        score_batch_split_kernel<float, false><<<grid, block, 0, stream>>>(p);
-    }
+  int C = (f_stream || f_rows) ? 0 : split_cluster(p.n_rows, sms);
+  if (f_split) {
+    const int want = atoi(force + 5);
+    if (want == 1 || want == 2 || want == 4 || want == 8) C = want;
+    else if (C == 0) C = 2;
+  }
+  if (C > 0 && p.V < 32 * (int64_t)C) C = f_split ? 1 : 0;  // a few logits per rank at least
+  if (C > 0) {
+    cudaError_t e;
+    if (dtype == STRIDE_DTYPE_BF16)
+      e = vec ? launch_split<__nv_bfloat16, true>(p, C, stream) : launch_split<__nv_bfloat16, false>(p, C, stream);
+    else
+      e = vec ? launch_split<float, true>(p, C, stream) : launch_split<float, false>(p, C, stream);
+    if (e != cudaSuccess) return e;
     return cudaGetLastError();
   }
   const int per_vec = dtype == STRIDE_DTYPE_BF16 ? 8 : 4;

@@ -22,10 +22,11 @@ def stride():
     return s
 
 
-@pytest.fixture(params=["auto", "stream", "split", "rows"])
+@pytest.fixture(params=["auto", "stream", "split", "split1", "split8", "rows"])
 def kernel(request, monkeypatch):
-    """Runs a test under each of the batch kernels (the library reads
-    STRIDE_BATCH_KERNEL on every call)."""
+    """Runs a test under each of the batch kernels, and the split kernel at
+    its automatic, smallest (one CTA per row) and largest (8-CTA) cluster
+    size (the library reads STRIDE_BATCH_KERNEL on every call)."""
     if request.param == "auto":
         monkeypatch.delenv("STRIDE_BATCH_KERNEL", raising=False)
     else:
