@@ -164,14 +164,14 @@ static __device__ ScanElem lookback(const BatchParams& p, int64_t tile, int lane
     uint32_t f = kStIncl;  // before row 0: never folded (tile 0 is inclusive)
     bool valid = idx >= 0;
     if (valid) {
-      f = ld_acquire_u32(p.flags + idx);
+      f = ld_acquire_u32(p.flags + idx * kFlagStride);
       while ((f & kStMask) == 0u) {
         if (globaltimer_ns() - t0 > p.timeout_ns) {
           f = kStIncl | kFlagTimedOut;
           break;
         }
         __nanosleep(64);
-        f = ld_acquire_u32(p.flags + idx);
+        f = ld_acquire_u32(p.flags + idx * kFlagStride);
       }
     }
     const bool is_incl = (f & kStMask) == kStIncl;
@@ -293,10 +293,10 @@ __device__ __forceinline__ RowCarry row_finalize(const BatchParams& p, int64_t t
       rc.incl.sl = e.fturn ? e.sl : sl0 + e.sl;
       rc.incl.fturn = 1;
     }
-    publish(p.incl + tile, p.flags + tile, rc.incl, kStIncl);
+    publish(p.incl + tile, p.flags + tile * kFlagStride, rc.incl, kStIncl);
   } else {
     rc.incl = e;
-    publish(p.agg + tile, p.flags + tile, e, kStAgg | (e.fturn ? kFlagTurnStart : 0u));
+    publish(p.agg + tile, p.flags + tile * kFlagStride, e, kStAgg | (e.fturn ? kFlagTurnStart : 0u));
   }
   return rc;
 }
@@ -324,7 +324,7 @@ __device__ __forceinline__ void row_resolve(const BatchParams& p, int64_t tile, 
       incl = combine(excl, rc.e);
       c_before = excl.c;
       st_before = rc.e.fturn ? 0.0 : excl.st;
-      publish(p.incl + tile, p.flags + tile, incl, kStIncl);
+      publish(p.incl + tile, p.flags + tile * kFlagStride, incl, kStIncl);
     }
   }
   if (lane != 0) return;

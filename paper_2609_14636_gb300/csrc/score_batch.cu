@@ -227,7 +227,7 @@ BatchWorkspaceLayout batch_workspace_layout(int64_t n_rows) {
   const size_t n = n_rows > 0 ? (size_t)n_rows : 0;
   L.ticket_off = 0;
   L.flags_off = 256;
-  L.agg_off = L.flags_off + up(n * sizeof(uint32_t));
+  L.agg_off = L.flags_off + up(n * sizeof(uint32_t) * kFlagStride);
   L.incl_off = L.agg_off + up(n * sizeof(ScanSlot));
   L.total = L.incl_off + up(n * sizeof(ScanSlot));
   L.clear_bytes = L.agg_off;  // ticket + flags
