@@ -114,6 +114,24 @@ def test_steps_small(stride, mode, lam, V, ld):
     _check_final(g, o, mode, lam)
 
 
+@pytest.mark.parametrize("B,V,ld", [(1, 4099, 4104), (3, 100, 104), (2, 9, 9), (5, 64, 64), (1500, 40, 40)])
+def test_steps_tiny_problems(stride, B, V, ld):
+    """One rollout, rows of one vector plus a tail, scalar rows, and more
+    rollouts than a wave of clusters holds."""
+    import torch
+
+    ring, steps = 2, 40
+    S, T, tok, Sp, Tp = _ring(B * 7 + V, ring, B, V, ld)
+    o_rows = oracle.row_logprobs(S, T, tok)
+    rng = np.random.default_rng(2)
+    turn_end = (rng.random((steps, B)) < 1 / 6).astype(np.uint8)
+    St, Tt = to_dev(Sp), to_dev(Tp)
+    tk = torch.from_numpy(tok).cuda()
+    g, o, worst = run_steps(stride, St, Tt, tk, turn_end, ring, B, 0, -25.0, V, check_every=1, o_rows=o_rows)
+    assert worst <= LOGP_ATOL
+    _check_final(g, o, 0, -25.0)
+
+
 def test_step_full_decode_workload(stride):
     """B=256 rollouts x 4,096 steps, V=151,936 bf16, a ring of 16 distinct
     step slabs (more bytes than L2), turn ends every U{96..768} steps, stopped
