@@ -240,7 +240,8 @@ def load_lambda(w) -> np.ndarray:
     return np.full(w.layout.n_traj, np.float32(synth.workload_lambda(w.name)), np.float32)
 
 
-WORKLOADS = ("batch_scoring", "long_agentic", "multi_teacher", "decode_step", "select", "tiny_reference")
+WORKLOADS = ("batch_scoring", "long_agentic", "multi_teacher", "decode_step", "select", "tiny_reference",
+             "vocab_parallel")
 
 
 def main() -> None:
@@ -265,6 +266,8 @@ def main() -> None:
         run_tiny(args)
     elif args.workload == "select":
         run_select(args)
+    elif args.workload == "vocab_parallel":
+        run_vocab_parallel(args)
     else:
         run_batch(args)
 
@@ -486,6 +489,108 @@ def run_batch(args) -> None:
         print(json.dumps(line), flush=True)
     if ws > 1:
         dist.destroy_process_group()
+
+
+def run_vocab_parallel(args, n_shards: int = 4) -> None:
+    """The batch-scoring workload with its logits split by vocabulary into
+    n_shards column shards, as a tensor-parallel teacher and student would
+    hold them: stride_partial_lse on every shard (each shard a column range
+    of the resident [rows, V] buffers, row stride V), stride_combine_partials,
+    stride_scan_logprobs.  On one GPU the shards run one after another, so a
+    step reads the same logit bytes as the fused path."""
+    import torch
+
+    ws, rank, local, dev = _setup_rank()
+    import paper_2609_14636_gb300 as stride
+    import synth
+
+    w = synth.batch_scoring()
+    lay = w.layout
+    if args.max_rows > 0:
+        lay = synth.sub_layout(lay, synth.first_trajectories(lay, args.max_rows))
+    R, V = lay.rows, w.recipe.V
+    lam = load_lambda(w)[: lay.n_traj]
+    S = torch.empty((R, V), dtype=torch.bfloat16, device=dev)
+    T = torch.empty((R, V), dtype=torch.bfloat16, device=dev)
+    tok = torch.empty(R, dtype=torch.int32, device=dev)
+    for r0 in range(0, R, 8192):
+        r1 = min(R, r0 + 8192)
+        synth.generate_rows(w.recipe, r0, r1 - r0, device=dev, out_S=S[r0:r1], out_T=T[r0:r1], out_tok=tok[r0:r1])
+    offs = [torch.from_numpy(a).to(dev) for a in (lay.traj_row_off, lay.turn_row_off, lay.traj_turn_off)]
+    lam_d = torch.from_numpy(lam).to(dev)
+    st = stride.new_state(lay.n_traj, dev)
+    ts = stride.new_turn_stats(lay.n_turns, dev)
+    parts = torch.empty((n_shards, R, 6), dtype=torch.float32, device=dev)
+    lps, lpt, opd = (torch.empty(R, dtype=torch.float32, device=dev) for _ in range(3))
+    status = torch.zeros(1, dtype=torch.int32, device=dev)
+    wsb = torch.empty(stride.stride_score_batch_workspace_size(R), dtype=torch.uint8, device=dev)
+    # shard k: columns [cuts[k], cuts[k+1]), cut on 16-byte boundaries
+    cuts = [((V * k // n_shards) // 8) * 8 for k in range(n_shards)] + [V]
+    stream = torch.cuda.current_stream()
+    evs = [torch.cuda.Event(enable_timing=True) for _ in range(4)]
+
+    def step(timed=False):
+        stride.stride_state_init(st, lay.n_traj, stream)
+        if timed:
+            evs[0].record(stream)
+        for k in range(n_shards):
+            c0, c1 = cuts[k], cuts[k + 1]
+            stride.stride_partial_lse(S[:, c0:c1], T[:, c0:c1], tok, c0, parts[k], dev_status=status, stream=stream)
+        if timed:
+            evs[1].record(stream)
+        stride.stride_combine_partials(parts, logp_s=lps, logp_t=lpt, dev_status=status, stream=stream)
+        if timed:
+            evs[2].record(stream)
+        stride.stride_scan_logprobs(lps, lpt, *offs, 0, R, stride.TURN_MEAN, lam_d, st, opd=opd, turn_stats=ts,
+                                    dev_status=status, workspace=wsb, stream=stream)
+        if timed:
+            evs[3].record(stream)
+
+    for _ in range(max(3, args.warmup)):
+        step()
+    torch.cuda.synchronize()
+    if int(status.item()) != 0:
+        raise RuntimeError(f"device status {int(status.item())}")
+    steps = max(1, min(args.steps, 30))
+    t_part, t_comb, t_scan = [], [], []
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with ClockSampler(local) as clk:
+        time.sleep(0.25)
+        e0.record(stream)
+        for _ in range(steps):
+            step(timed=True)
+            torch.cuda.synchronize()
+            t_part.append(evs[0].elapsed_time(evs[1]))
+            t_comb.append(evs[1].elapsed_time(evs[2]))
+            t_scan.append(evs[2].elapsed_time(evs[3]))
+        e1.record(stream)
+        torch.cuda.synchronize()
+        time.sleep(0.05)
+    ms_step = max_over_ranks(statistics.mean(a + b + c for a, b, c in zip(t_part, t_comb, t_scan)), dev)
+    peaks = measured_peaks()
+    peak = peaks.get("hbm_gbs", 6800.0)
+    part_bytes = R * (2 * V * 2 + n_shards * (4 + 24))  # every shard's logits, tokens, partials written
+    part_ms = statistics.mean(t_part)
+    achieved = part_bytes / (part_ms * 1e-3) / 1e9
+    if rank == 0:
+        line = _common_line(args, ws, ms_step, whole_job_rate(R, ws, ms_step))
+        line.update({
+            "config": {"workload": f"{w.name} in {n_shards} vocabulary shards", "rows": R, "vocab": V,
+                       "shards": n_shards, "shard_columns": [cuts[k + 1] - cuts[k] for k in range(n_shards)],
+                       "stop_mode": "turn_mean", "lambda": float(lam[0]),
+                       "l2": f"inputs ({2 * R * V * 2 / 1e9:.1f} GB) larger than L2 (129 MB): no flush",
+                       "timing": "per step: the shards' partial passes, the combine and the scan, each "
+                                 "bracketed by CUDA events; the step is their sum (state init excluded)"},
+            "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s", "frac": achieved / peak,
+                         "traffic": None, "algorithmic_bytes_per_launch": part_bytes / n_shards,
+                         "kernel": "partial_lse_kernel<bf16> (one CTA per row and shard)",
+                         "ms_partials": part_ms, "ms_combine": statistics.mean(t_comb),
+                         "ms_scan": statistics.mean(t_scan),
+                         "peak_source": "MEASURED_PEAKS.json hbm_gbs (of measured)" if "hbm_gbs" in peaks
+                         else "fallback 6.8 TB/s"},
+            "clocks": clk.summary(), "gpu_launches": steps * (1 + n_shards + 2),
+        })
+        print(json.dumps(line), flush=True)
 
 
 def _graph(fn):

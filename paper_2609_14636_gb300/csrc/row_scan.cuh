@@ -312,6 +312,14 @@ __device__ __forceinline__ RowCarry row_finalize(const BatchParams& p, int64_t t
 // (c_before - st_before / n_k).  The sums are monotone, so this selects
 // exactly the rows up to the first crossing (its turn, in turn mode).
 // rc is read in lane 0.
+// row_tail is the single-thread part once the row's inclusive prefix is
+// known: incl (running sum and open-turn sums through the row), c_before
+// and st_before (the running sum and open turn's sum of log pi_T before it);
+// of rc only rc.e.sl (the row's loss term) is read.
+__device__ __forceinline__ void row_tail(const BatchParams& p, int64_t r, const RowMeta& meta,
+                                         const RowCarry& rc, const ScanElem& incl, double c_before,
+                                         double st_before, bool timed_out);
+
 __device__ __forceinline__ void row_resolve(const BatchParams& p, int64_t tile, int64_t r,
                                             const RowMeta& meta, RowCarry rc, int lane) {
   const int seeded = __shfl_sync(0xffffffffu, rc.seeded, 0);
@@ -328,6 +336,12 @@ __device__ __forceinline__ void row_resolve(const BatchParams& p, int64_t tile, 
     }
   }
   if (lane != 0) return;
+  row_tail(p, r, meta, rc, incl, c_before, st_before, timed_out);
+}
+
+__device__ __forceinline__ void row_tail(const BatchParams& p, int64_t r, const RowMeta& meta,
+                                         const RowCarry& rc, const ScanElem& incl, double c_before,
+                                         double st_before, bool timed_out) {
   if (timed_out) set_status(p.dev_status, STRIDE_DEV_TIMEOUT);
   if (meta.bad) return;
   const int64_t n_k = meta.turn_end - meta.turn_start;

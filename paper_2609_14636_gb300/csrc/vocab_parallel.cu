@@ -9,8 +9,8 @@
 // into the row's log-sum-exp (combine_kernel), which gives the same
 // log-probs as the full row.  The rest of the path (turn statistics, stop
 // rule, OPD loss, profile, carried state) then runs on the log-probs
-// (scan_logprobs_kernel), one warp per row with the same decoupled-lookback
-// protocol as the fused kernels (row_scan.cuh).
+// (scan_logprobs_tile_kernel): a segmented scan per tile of 256 rows, and
+// the fused kernels' decoupled lookback (row_scan.cuh) between tiles.
 #include <math.h>
 
 #include "row_scan.cuh"
@@ -113,29 +113,280 @@ __global__ void combine_kernel(const float* __restrict__ parts, int32_t n_shards
   if (lse_t) lse_t[r] = lt;
 }
 
-// One warp per row, rows taken in ticket order: trajectory/turn lookup, the
-// row's element (from the given log-probs), the lookback and the row tail.
-constexpr int kScanWarpsPerCta = 8;
-__global__ void __launch_bounds__(32 * kScanWarpsPerCta) scan_logprobs_kernel(const BatchParams p,
-                                                                             const float* logp_s,
-                                                                             const float* logp_t) {
-  const int lane = threadIdx.x & 31;
-  uint32_t t = 0;
-  if (lane == 0) t = atomicAdd(p.ticket, 1u);
-  t = __shfl_sync(0xffffffffu, t, 0);
-  if ((int64_t)t >= p.n_rows) return;
-  const int64_t tile = t;
-  const int64_t r = p.row_begin + tile;
-  float ls = 0.f, lt = 0.f;
-  if (lane == 0) {
-    ls = __ldg(logp_s + tile);
-    lt = __ldg(logp_t + tile);
-    validate_layout(p, tile);
+// The scan on given log-probs, one tile of kScanTileRows consecutive rows per
+// CTA (one row per thread), tiles taken in ticket order.  Without a logit
+// pass to hide it, a lookback per row is what the time goes to (each row
+// waits on its predecessors' prefixes), so the rows of a tile are scanned
+// together in the CTA and only the tile takes part in the decoupled
+// lookback:
+//   1. warp 0 finds the tile's first turn and trajectory; the CTA stages the
+//      offsets of the next kScanTileRows + 1 turns and trajectories in shared
+//      memory and every thread finds its row's turn and trajectory there;
+//   2. each row's element: the stop-sum term, log pi_T, d, logp_S * d, and
+//      two restart marks -- the open-turn sums restart at a turn's first row,
+//      the running sum at a seeded row (a trajectory's first row, or the
+//      window's), whose element already holds the carried state;
+//   3. a segmented inclusive scan of the tile's elements (warp shuffles, then
+//      the warps' totals);
+//   4. the tile's aggregate is published (as an INCLUSIVE prefix at once if
+//      the tile holds a seeded row, since nothing before it matters then;
+//      tile 0 always does), warp 0 folds its predecessors' (row_scan.cuh
+//      lookback) and publishes the tile's inclusive prefix;
+//   5. every row completes with its inclusive and exclusive prefixes: turn
+//      statistics, stop test, retained loss, carried state (row_tail), and
+//      the within-turn profile into the CTA's shared bins.
+constexpr int kScanTileRows = 256;
+constexpr int kScanTileWarps = kScanTileRows / 32;
+constexpr int kRestartTurn = 1;  // st, sd, sl restart at this row
+constexpr int kRestartSum = 2;   // c restarts (a seeded row)
+
+struct TileElem {
+  double c, st, sd, sl;
+  int flags;
+};
+
+__device__ __forceinline__ TileElem tile_combine(const TileElem& a, const TileElem& b) {
+  TileElem r;
+  r.c = (b.flags & kRestartSum) ? b.c : a.c + b.c;
+  r.st = (b.flags & kRestartTurn) ? b.st : a.st + b.st;
+  r.sd = (b.flags & kRestartTurn) ? b.sd : a.sd + b.sd;
+  r.sl = (b.flags & kRestartTurn) ? b.sl : a.sl + b.sl;
+  r.flags = a.flags | b.flags;
+  return r;
+}
+
+__device__ __forceinline__ TileElem tile_shfl_up(const TileElem& v, int d) {
+  TileElem o;
+  o.c = __shfl_up_sync(0xffffffffu, v.c, d);
+  o.st = __shfl_up_sync(0xffffffffu, v.st, d);
+  o.sd = __shfl_up_sync(0xffffffffu, v.sd, d);
+  o.sl = __shfl_up_sync(0xffffffffu, v.sl, d);
+  o.flags = __shfl_up_sync(0xffffffffu, v.flags, d);
+  return o;
+}
+
+// Largest j in [0, n) with a[j] <= r (a ascending, a[0] <= r).
+__device__ __forceinline__ int smem_upper_le(const int64_t* a, int n, int64_t r) {
+  int lo = 0, hi = n - 1;
+  while (lo < hi) {
+    const int mid = (lo + hi + 1) >> 1;
+    if (a[mid] <= r) lo = mid; else hi = mid - 1;
   }
-  const RowMeta meta = find_row_meta(p, r, lane);
-  RowCarry rc;
-  if (lane == 0) rc = row_finalize(p, tile, r, meta, true, ls, lt, 0.f, 0.f, p.profile, true);
-  row_resolve(p, tile, r, meta, rc, lane);
+  return lo;
+}
+
+__global__ void __launch_bounds__(kScanTileRows) scan_logprobs_tile_kernel(const BatchParams p,
+                                                                          const float* __restrict__ logp_s,
+                                                                          const float* __restrict__ logp_t,
+                                                                          int64_t n_tiles) {
+  __shared__ int64_t s_turn_off[kScanTileRows + 1];
+  __shared__ int64_t s_traj_turn[kScanTileRows + 1];  // traj_turn_off, widened
+  __shared__ int64_t s_first[2];                      // first turn, first trajectory of the tile
+  __shared__ TileElem s_wtot[kScanTileWarps];
+  __shared__ TileElem s_excl;
+  __shared__ TileElem s_agg;
+  __shared__ int s_flags;  // bit 0: lookback timed out
+  __shared__ double s_prof[3 * STRIDE_PROFILE_BINS];
+  __shared__ int64_t s_tile;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  if (tid == 0) s_tile = (int64_t)atomicAdd(p.ticket, 1u);
+  if (tid < 3 * STRIDE_PROFILE_BINS) s_prof[tid] = 0.0;
+  __syncthreads();
+  const int64_t tile = s_tile;
+  if (tile >= n_tiles) return;
+  const int64_t t0 = tile * kScanTileRows;           // first window row of the tile
+  const int64_t n_here = min((int64_t)kScanTileRows, p.n_rows - t0);
+  const int64_t r0 = p.row_begin + t0;
+
+  // Layout checks, spread over every thread of the launch.
+  {
+    bool bad = false;
+    const int64_t stride = n_tiles * kScanTileRows;
+    for (int64_t k = t0 + tid; k < p.n_turns; k += stride)
+      bad |= __ldg(p.turn_row_off + k + 1) <= __ldg(p.turn_row_off + k);
+    for (int64_t i = t0 + tid; i < p.n_traj; i += stride) {
+      const int32_t a = __ldg(p.traj_turn_off + i), b = __ldg(p.traj_turn_off + i + 1);
+      if (a < 0 || b < a || b > p.n_turns) {
+        bad = true;
+      } else {
+        bad |= __ldg(p.turn_row_off + a) != __ldg(p.traj_row_off + i);
+        bad |= __ldg(p.turn_row_off + b) != __ldg(p.traj_row_off + i + 1);
+      }
+    }
+    if (bad) set_status(p.dev_status, STRIDE_DEV_BAD_LAYOUT);
+  }
+
+  // 1. the tile's first turn and trajectory, then the staged offsets
+  if (warp == 0) {
+    const bool ok = p.n_turns > 0 && __ldg(p.turn_row_off) <= r0 && __ldg(p.traj_turn_off) <= 0;
+    int64_t k0 = 0, i0 = 0;
+    if (ok) {
+      k0 = warp_upper_le(p.turn_row_off, 0, p.n_turns - 1, r0, lane);
+      // trajectory holding turn k0: largest i with traj_turn_off[i] <= k0
+      int64_t lo = 0, hi = p.n_traj - 1;
+      while (hi > lo) {
+        const int64_t step = (hi - lo + 31) / 32;
+        const int64_t q = lo + step * (lane + 1);
+        const bool le = (q <= hi) && ((int64_t)__ldg(p.traj_turn_off + q) <= k0);
+        const int k = __popc(__ballot_sync(0xffffffffu, le));
+        const int64_t nlo = lo + step * k;
+        const int64_t nhi = (k < 32) ? min(hi, lo + step * (k + 1) - 1) : hi;
+        lo = nlo;
+        hi = nhi;
+      }
+      i0 = lo;
+    }
+    if (lane == 0) {
+      s_first[0] = ok ? k0 : -1;
+      s_first[1] = i0;
+    }
+  }
+  __syncthreads();
+  const int64_t k0 = s_first[0], i0 = s_first[1];
+  if (k0 >= 0) {
+    for (int j = tid; j <= kScanTileRows; j += kScanTileRows) {
+      s_turn_off[j] = __ldg(p.turn_row_off + min(k0 + j, (int64_t)p.n_turns));
+      s_traj_turn[j] = __ldg(p.traj_turn_off + min(i0 + j, (int64_t)p.n_traj));
+    }
+  }
+  __syncthreads();
+
+  // 2. this thread's row and its element
+  const int64_t w = t0 + tid;  // window row
+  const int64_t r = p.row_begin + w;
+  const bool live = tid < n_here;
+  RowMeta meta;
+  meta.bad = true;
+  meta.traj = 0;
+  meta.turn = 0;
+  meta.local_turn = 0;
+  meta.traj_start = meta.traj_end = meta.turn_start = meta.turn_end = 0;
+  if (live && k0 >= 0) {
+    const int nk = (int)min((int64_t)kScanTileRows, (int64_t)p.n_turns - k0);
+    const int j = smem_upper_le(s_turn_off, nk, r);
+    const int64_t turn = k0 + j;
+    const int ni = (int)min((int64_t)kScanTileRows, (int64_t)p.n_traj - i0);
+    const int q = smem_upper_le(s_traj_turn, ni, turn);
+    const int64_t traj = i0 + q;
+    meta.turn = (int32_t)turn;
+    meta.traj = (int32_t)traj;
+    meta.turn_start = s_turn_off[j];
+    meta.turn_end = s_turn_off[j + 1];
+    meta.local_turn = (int32_t)(turn - s_traj_turn[q]);
+    meta.traj_start = __ldg(p.traj_row_off + traj);
+    meta.traj_end = __ldg(p.traj_row_off + traj + 1);
+    meta.bad = !(meta.turn_start <= r && r < meta.turn_end) || !(meta.traj_start <= r && r < meta.traj_end) ||
+               !(s_traj_turn[q] <= turn && turn < s_traj_turn[q + 1]) || j + 1 > kScanTileRows;
+  }
+  TileElem x = {0.0, 0.0, 0.0, 0.0, 0};
+  double c_before = 0.0, st_before = 0.0, e_sl = 0.0;
+  int fturn = 0;
+  if (live) {
+    const float nan = __int_as_float(0x7fc00000);
+    float lps = __ldg(logp_s + w), lpt = __ldg(logp_t + w);
+    if (meta.bad) {
+      set_status(p.dev_status, STRIDE_DEV_BAD_LAYOUT);
+      lps = nan;
+      lpt = nan;
+    }
+    const float dd = lps - lpt;
+    if (p.out.opd) p.out.opd[w] = dd;
+    const int64_t n_k = meta.turn_end - meta.turn_start;
+    const double ec = (p.mode == STRIDE_STOP_TURN_MEAN) ? (double)lpt / (double)(n_k > 0 ? n_k : 1) : (double)lpt;
+    const double est = (double)lpt, esd = (double)dd, esl = (double)lps * (double)dd;
+    e_sl = esl;
+    fturn = (r == meta.turn_start) ? 1 : 0;
+    if (p.profile && !meta.bad) {
+      const int jb = (int)((10 * (r - meta.turn_start)) / n_k);  // Observation 1 decile
+      atomicAdd(s_prof + 3 * jb + 0, esd);
+      atomicAdd(s_prof + 3 * jb + 1, est);
+      atomicAdd(s_prof + 3 * jb + 2, 1.0);
+    }
+    const bool seeded = (w == 0) || (r == meta.traj_start) || meta.bad;
+    if (seeded && !meta.bad) {
+      const stride_scan_state* sp = p.state + meta.traj;
+      const double cum0 = __ldcg(&sp->cum);
+      const double st0 = fturn ? 0.0 : __ldcg(&sp->turn_sum_t);
+      const double sd0 = fturn ? 0.0 : __ldcg(&sp->turn_sum_d);
+      const double sl0 = fturn ? 0.0 : __ldcg(&sp->turn_sum_l);
+      x = TileElem{cum0 + ec, st0 + est, sd0 + esd, sl0 + esl, kRestartSum | kRestartTurn};
+      c_before = cum0;
+      st_before = st0;
+    } else if (seeded) {
+      x = TileElem{ec, est, esd, esl, kRestartSum | kRestartTurn};  // NaN: nothing after a bad row is meaningful
+    } else {
+      x = TileElem{ec, est, esd, esl, fturn ? kRestartTurn : 0};
+    }
+    if (seeded) x.flags |= 4;  // bit 2: this row's exclusive prefix is the carried state, not the scan
+  }
+
+  // 3. segmented inclusive scan over the tile
+  TileElem incl = x;
+#pragma unroll
+  for (int d = 1; d < 32; d <<= 1) {
+    const TileElem o = tile_shfl_up(incl, d);
+    if (lane >= d) incl = tile_combine(o, incl);
+  }
+  TileElem excl_in_warp = tile_shfl_up(incl, 1);
+  if (lane == 31) s_wtot[warp] = incl;
+  __syncthreads();
+  TileElem wpre = {0.0, 0.0, 0.0, 0.0, 0};
+  for (int v = 0; v < warp; ++v) wpre = tile_combine(wpre, s_wtot[v]);
+  const TileElem tile_incl = tile_combine(wpre, incl);
+  const TileElem tile_excl = (lane == 0) ? wpre : tile_combine(wpre, excl_in_warp);
+
+  // 4. publish the tile's aggregate, fold predecessors, publish its prefix
+  if (tid == (int)(n_here - 1)) {
+    ScanElem agg{tile_incl.c, tile_incl.st, tile_incl.sd, tile_incl.sl, tile_incl.flags & kRestartTurn};
+    if (tile_incl.flags & kRestartSum) {
+      publish(p.incl + tile, p.flags + tile * kFlagStride, agg, kStIncl);
+    } else {
+      publish(p.agg + tile, p.flags + tile * kFlagStride, agg,
+              kStAgg | ((tile_incl.flags & kRestartTurn) ? kFlagTurnStart : 0u));
+    }
+    s_agg = tile_incl;  // the aggregate, for warp 0 below
+  }
+  __syncthreads();
+  if (warp == 0) {
+    const TileElem agg = s_agg;
+    TileElem pre = {0.0, 0.0, 0.0, 0.0, 0};
+    bool timed_out = false;
+    // The rows before the tile's first seeded row need the predecessors' sum
+    // (a tile whose first row is seeded needs nothing).
+    if (!(__shfl_sync(0xffffffffu, x.flags, 0) & kRestartSum)) {
+      const ScanElem e = lookback(p, tile, lane, timed_out);
+      pre = TileElem{e.c, e.st, e.sd, e.sl, 0};
+      if (lane == 0 && !(agg.flags & kRestartSum)) {
+        const TileElem inc = tile_combine(pre, agg);
+        ScanElem ie{inc.c, inc.st, inc.sd, inc.sl, 1};
+        publish(p.incl + tile, p.flags + tile * kFlagStride, ie, kStIncl);
+      }
+    }
+    if (lane == 0) {
+      s_excl = pre;
+      s_flags = timed_out ? 1 : 0;
+    }
+  }
+  __syncthreads();
+
+  // 5. complete every row
+  if (live) {
+    const TileElem pre = s_excl;
+    const TileElem ri = tile_combine(pre, tile_incl);
+    if (!(x.flags & 4)) {
+      const TileElem re = tile_combine(pre, tile_excl);
+      c_before = re.c;
+      st_before = fturn ? 0.0 : re.st;
+    }
+    RowCarry rc;
+    rc.e = ScanElem{0.0, 0.0, 0.0, e_sl, fturn};
+    const ScanElem si{ri.c, ri.st, ri.sd, ri.sl, 1};
+    row_tail(p, r, meta, rc, si, c_before, st_before, (s_flags & 1) != 0);
+  }
+  if (p.profile) {
+    __syncthreads();
+    if (tid < 3 * STRIDE_PROFILE_BINS && s_prof[tid] != 0.0) atomicAdd(p.profile + tid, s_prof[tid]);
+  }
 }
 
 cudaError_t launch_partial_lse(const void* S, const void* T, int dtype, bool vec, int64_t ld,
@@ -167,8 +418,8 @@ cudaError_t launch_combine_partials(const float* parts, int32_t n_shards, int64_
 
 cudaError_t launch_scan_logprobs(const BatchParams& p, const float* logp_s, const float* logp_t,
                                  cudaStream_t stream) {
-  const unsigned grid = (unsigned)((p.n_rows + kScanWarpsPerCta - 1) / kScanWarpsPerCta);
-  scan_logprobs_kernel<<<grid, 32 * kScanWarpsPerCta, 0, stream>>>(p, logp_s, logp_t);
+  const int64_t n_tiles = (p.n_rows + kScanTileRows - 1) / kScanTileRows;
+  scan_logprobs_tile_kernel<<<(unsigned)n_tiles, kScanTileRows, 0, stream>>>(p, logp_s, logp_t, n_tiles);
   return cudaGetLastError();
 }
 

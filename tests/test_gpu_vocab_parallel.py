@@ -112,6 +112,43 @@ def test_scan_on_sharded_logprobs(stride, mode):
     compare_scan(g, o, lay, mode, lam)
 
 
+def _tile_layout(kind, rng):
+    if kind == "one_row_turns":  # hundreds of turns inside one 256-row tile
+        turns = [[int(x) for x in rng.choice([1, 1, 1, 2, 5, 40], size=180)] for _ in range(3)]
+    else:  # trajectories spanning dozens of tiles
+        turns = [[int(x) for x in rng.integers(64, 513, size=30)] for _ in range(3)]
+    return synth.layout_from_turn_lengths(turns)
+
+
+@pytest.mark.parametrize("kind", ["one_row_turns", "long_trajectories"])
+@pytest.mark.parametrize("mode", [0, 1])
+def test_scan_tiles_on_logprobs(stride, kind, mode):
+    """stride_scan_logprobs on given log-probs against the oracle's scan of
+    the same values: many one-row turns per tile, trajectories across many
+    tiles, and windows that cut tiles, trajectories and turns."""
+    import torch
+
+    rng = np.random.default_rng(63 + mode)
+    lay = _tile_layout(kind, rng)
+    R = lay.rows
+    lt = (-np.abs(rng.standard_normal(R) * 2.0) - 0.5).astype(np.float32)
+    ls = (lt + rng.standard_normal(R).astype(np.float32) * np.float32(0.3)).astype(np.float32)
+    d = (ls - lt).astype(np.float32)  # as the kernel forms it
+    o0 = oracle.scan_batch(lt.astype(np.float64), d.astype(np.float64), lay.traj_row_off, lay.turn_row_off,
+                           lay.traj_turn_off, mode, np.float64(-1e30), logp_s=ls.astype(np.float64))
+    lam = np.float32(np.median(o0["turn_cum"]) if mode == 0 else np.median(o0["row_cum"]))
+    o = oracle.scan_batch(lt.astype(np.float64), d.astype(np.float64), lay.traj_row_off, lay.turn_row_off,
+                          lay.traj_turn_off, mode, np.float64(lam), logp_s=ls.astype(np.float64))
+    o.update(logp_t=lt.astype(np.float64), d=d.astype(np.float64), logp_s=ls.astype(np.float64))
+    ls_d, lt_d = torch.from_numpy(ls).cuda(), torch.from_numpy(lt).cuda()
+    for windows in (None, [(0, 777), (777, R // 2 + 13), (R // 2 + 13, R)]):
+        g = _scan(stride, ls_d, lt_d, lay, mode, lam, windows)
+        assert g["status"] == 0
+        assert np.array_equal(g["opd"], d)
+        compare_scan(g, o, lay, mode, lam)
+    assert int(np.sum(o["stop_row"] >= 0)) > 0
+
+
 def test_token_owned_by_no_shard(stride):
     import torch
 
