@@ -319,7 +319,7 @@ STRIDE_API int stride_select_restart(const float* turn_mean, const int32_t* n_tu
  * implicit device synchronisation of cudaMalloc/cudaFree, or because they
  * were handed only inputs and outputs.  This entry point takes the same
  * arguments minus the workspace and uses a fixed scratch array that the
- * library holds on every device that loads it (about 12.6 MB) until the
+ * library holds on every device that loads it (about 13.1 MB) until the
  * process exits.  It allocates nothing.
  *
  * - Windows of more than STRIDE_NOALLOC_MAX_ROWS rows return

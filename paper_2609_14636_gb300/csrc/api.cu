@@ -148,6 +148,8 @@ int prepare_batch(stride::BatchParams& p, stride::BatchWorkspaceLayout& L, const
   p.flags = reinterpret_cast<uint32_t*>(ws + L.flags_off);
   p.agg = reinterpret_cast<stride::ScanSlot*>(ws + L.agg_off);
   p.incl = reinterpret_cast<stride::ScanSlot*>(ws + L.incl_off);
+  p.ws_logp_s = reinterpret_cast<float*>(ws + L.logp_s_off);
+  p.ws_logp_t = reinterpret_cast<float*>(ws + L.logp_t_off);
   p.timeout_ns = 2000000000ull;  // 2 s bound on any single device-side wait
   return STRIDE_OK;
 }

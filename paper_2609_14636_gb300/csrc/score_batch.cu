@@ -91,11 +91,16 @@ __global__ void __launch_bounds__(kBatchThreads, 2) score_batch_kernel(const Bat
 // (each SM streams its rows one after another), so a window of at most 8
 // rows per SM splits every row over the C CTAs of a thread-block cluster
 // instead (C = 1: one CTA per row), C chosen at launch (split_cluster below)
-// so that the window is one wave of 128-thread CTAs.  Rank 0 takes the row's
-// ticket and shares it through distributed shared memory; every rank streams
-// its share of the vocabulary of S and T; rank 0 merges the ranks' pairs,
-// then runs the row tail (finalize, lookback, resolve) after the other ranks
-// have left.
+// so that the window is one wave of 128-thread CTAs.  Cluster i scores
+// window row i: every rank streams its share of the vocabulary of S and T,
+// rank 0 merges the ranks' pairs through distributed shared memory, writes
+// the row's outputs and leaves its two log-probs in the workspace.  The scan
+// (turn statistics, stop rule, loss, profile, carried state) then runs as
+// the tiled scan on those log-probs (vocab_parallel.cu), launched as a
+// programmatic dependent of this kernel.  In a window whose rows all finish
+// streaming together, a lookback per row cost a chain of prefixes after the
+// last row (12 us on a 512-row segment); the tiled scan folds 256 rows per
+// step of that chain.
 namespace cg = cooperative_groups;
 constexpr int kSplitMaxCluster = 8;
 constexpr int kSplitThreads = 128;
@@ -107,31 +112,26 @@ __global__ void __launch_bounds__(kSplitThreads, kSplitBlocksPerSm)
     score_batch_split_kernel(const BatchParams p) {
   __shared__ float s_red[4][kSplitWarps];
   __shared__ float s_part[4];
-  __shared__ int64_t s_tile;
+  // the dependent scan may be scheduled once every CTA of this grid runs
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
   cg::cluster_group cluster = cg::this_cluster();
   const int rank = (int)cluster.block_rank();
   const int n_ranks = (int)cluster.num_blocks();
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  if (rank == 0 && tid == 0) s_tile = (int64_t)atomicAdd(p.ticket, 1u);
-  cluster.sync();
-  const int64_t tile = *cluster.map_shared_rank(&s_tile, 0);
-  const int64_t r = p.row_begin + tile;
+  const int64_t tile = blockIdx.x / n_ranks;  // window row
   const LT* srow = reinterpret_cast<const LT*>(p.S) + tile * p.ld;
   const LT* trow = teacher_row<LT>(p, tile);
 
   int32_t y = 0;
   float xs = __int_as_float(0x7fc00000), xt = xs;
-  RowMeta meta;
-  if (rank == 0 && warp == 0) {
-    if (lane == 0) {
-      y = __ldg(p.tokens + tile);
-      if (y >= 0 && y < p.V) {
-        xs = to_f32(srow[y]);
-        xt = to_f32(trow[y]);
-      }
-      validate_layout(p, tile);
+  if (rank == 0 && tid == 0) {
+    y = __ldg(p.tokens + tile);
+    if (y >= 0 && y < p.V) {
+      xs = to_f32(srow[y]);
+      xt = to_f32(trow[y]);
     }
-    meta = find_row_meta(p, r, lane);
+  } else if (rank == 0 && tid == 32) {
+    validate_layout(p, tile);  // this row's share of the layout checks (the scan skips them)
   }
   int c0, c1;
   if (VEC) {
@@ -182,10 +182,22 @@ __global__ void __launch_bounds__(kSplitThreads, kSplitBlocksPerSm)
       sT = peer[3];
     }
     warp_merge2(mS, sS, mT, sT);
+    if (lane == 0) {
+      const float lse_s = lse_finish(mS, sS), lse_t = lse_finish(mT, sT);
+      if (!(y >= 0 && y < p.V)) set_status(p.dev_status, STRIDE_DEV_TOKEN_RANGE);
+      const float lps = xs - lse_s, lpt = xt - lse_t;
+      const stride_row_outputs& o = p.out;
+      if (o.logp_s) o.logp_s[tile] = lps;
+      if (o.logp_t) o.logp_t[tile] = lpt;
+      if (o.lse_s) o.lse_s[tile] = lse_s;
+      if (o.lse_t) o.lse_t[tile] = lse_t;
+      if (o.x_s) o.x_s[tile] = xs;
+      if (o.x_t) o.x_t[tile] = xt;
+      p.ws_logp_s[tile] = lps;
+      p.ws_logp_t[tile] = lpt;
+    }
   }
   cluster.sync();  // the ranks' shared memory has been read: they may leave
-  if (rank != 0 || warp != 0) return;
-  finish_row(p, tile, r, meta, y, xs, xt, lse_finish(mS, sS), lse_finish(mT, sT), lane);
 }
 
 // Multi-teacher pre-pass: the teacher row of each window row, from its
@@ -229,7 +241,9 @@ BatchWorkspaceLayout batch_workspace_layout(int64_t n_rows) {
   L.flags_off = 256;
   L.agg_off = L.flags_off + up(n * sizeof(uint32_t) * kFlagStride);
   L.incl_off = L.agg_off + up(n * sizeof(ScanSlot));
-  L.total = L.incl_off + up(n * sizeof(ScanSlot));
+  L.logp_s_off = L.incl_off + up(n * sizeof(ScanSlot));
+  L.logp_t_off = L.logp_s_off + up(n * sizeof(float));
+  L.total = L.logp_t_off + up(n * sizeof(float));
   L.clear_bytes = L.agg_off;  // ticket + flags
   if (n == 0) L.total = 0;
   return L;
@@ -304,7 +318,11 @@ cudaError_t launch_score_batch(const BatchParams& p, int dtype, bool vec, cudaSt
     else
       e = vec ? launch_split<float, true>(p, C, stream) : launch_split<float, false>(p, C, stream);
     if (e != cudaSuccess) return e;
-    return cudaGetLastError();
+    // the scan on the rows' log-probs; its tile tickets use the header's
+    // second word (cleared with the first)
+    BatchParams q = p;
+    q.ticket = p.ticket + 1;
+    return launch_scan_logprobs(q, p.ws_logp_s, p.ws_logp_t, stream, true);
   }
   const int per_vec = dtype == STRIDE_DTYPE_BF16 ? 8 : 4;
   if (vec && p.V >= per_vec && !f_rows) return launch_score_batch_stream(p, dtype, stream);

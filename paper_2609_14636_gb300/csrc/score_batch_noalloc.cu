@@ -38,10 +38,11 @@ constexpr size_t up256(size_t x) { return (x + 255) & ~size_t(255); }
 
 // Same layout as stride_score_batch's workspace for STRIDE_NOALLOC_MAX_ROWS
 // rows: 256-byte header, one uint32 flag per 128-byte line, two 32-byte scan
-// slots per row (12.58 MB for 65,536 rows).
+// slots and two float log-probs per row (13.11 MB for 65,536 rows).
 constexpr size_t kNoAllocBytes =
     256 + up256(sizeof(uint32_t) * (size_t)stride::kFlagStride * (size_t)STRIDE_NOALLOC_MAX_ROWS) +
-    2 * up256(sizeof(stride::ScanSlot) * (size_t)STRIDE_NOALLOC_MAX_ROWS);
+    2 * up256(sizeof(stride::ScanSlot) * (size_t)STRIDE_NOALLOC_MAX_ROWS) +
+    2 * up256(sizeof(float) * (size_t)STRIDE_NOALLOC_MAX_ROWS);
 
 // The scratch.  In host code `g_noalloc_scratch` is only a handle for the
 // runtime: its device address comes from cudaGetSymbolAddress below.

@@ -50,6 +50,8 @@ struct BatchParams {
   uint32_t* flags;
   ScanSlot* agg;
   ScanSlot* incl;
+  float* ws_logp_s;  // per window row, written by the small-window kernel for the tiled scan
+  float* ws_logp_t;
   uint64_t timeout_ns;
 };
 
@@ -84,7 +86,7 @@ struct SelectParams {
 
 // Workspace layout of stride_score_batch (all offsets 256-byte aligned).
 struct BatchWorkspaceLayout {
-  size_t ticket_off, flags_off, agg_off, incl_off, clear_bytes, total;
+  size_t ticket_off, flags_off, agg_off, incl_off, logp_s_off, logp_t_off, clear_bytes, total;
 };
 BatchWorkspaceLayout batch_workspace_layout(int64_t n_rows);
 
@@ -119,7 +121,7 @@ cudaError_t launch_combine_partials(const float* parts, int32_t n_shards, int64_
                                     float* logp_t, float* lse_s, float* lse_t, int32_t* dev_status,
                                     cudaStream_t stream);
 cudaError_t launch_scan_logprobs(const BatchParams& p, const float* logp_s, const float* logp_t,
-                                 cudaStream_t stream);
+                                 cudaStream_t stream, bool dependent = false);
 cudaError_t launch_buffer_record(float* buf_mean, int32_t* buf_n_turns, int32_t n_tasks, int32_t T_max,
                                  const int32_t* task, const int32_t* k0, const stride_turn_stats* ts,
                                  const int32_t* traj_turn_off, int32_t n_traj, int32_t* dev_status,

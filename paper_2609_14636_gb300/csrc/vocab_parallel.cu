@@ -119,9 +119,10 @@ __global__ void combine_kernel(const float* __restrict__ parts, int32_t n_shards
 // waits on its predecessors' prefixes), so the rows of a tile are scanned
 // together in the CTA and only the tile takes part in the decoupled
 // lookback:
-//   1. warp 0 finds the tile's first turn and trajectory; the CTA stages the
-//      offsets of the next kScanTileRows + 1 turns and trajectories in shared
-//      memory and every thread finds its row's turn and trajectory there;
+//   1. warps 0 and 1 find the tile's first turn and trajectory; the CTA
+//      stages the offsets of the next kScanTileRows + 1 turns and
+//      trajectories in shared memory and every thread finds its row's turn
+//      and trajectory there;
 //   2. each row's element: the stop-sum term, log pi_T, d, logp_S * d, and
 //      two restart marks -- the open-turn sums restart at a turn's first row,
 //      the running sum at a seeded row (a trajectory's first row, or the
@@ -178,8 +179,9 @@ __device__ __forceinline__ int smem_upper_le(const int64_t* a, int n, int64_t r)
 __global__ void __launch_bounds__(kScanTileRows) scan_logprobs_tile_kernel(const BatchParams p,
                                                                           const float* __restrict__ logp_s,
                                                                           const float* __restrict__ logp_t,
-                                                                          int64_t n_tiles) {
+                                                                          int64_t n_tiles, bool validate) {
   __shared__ int64_t s_turn_off[kScanTileRows + 1];
+  __shared__ int64_t s_traj_row[kScanTileRows + 1];   // traj_row_off
   __shared__ int64_t s_traj_turn[kScanTileRows + 1];  // traj_turn_off, widened
   __shared__ int64_t s_first[2];                      // first turn, first trajectory of the tile
   __shared__ TileElem s_wtot[kScanTileWarps];
@@ -189,6 +191,9 @@ __global__ void __launch_bounds__(kScanTileRows) scan_logprobs_tile_kernel(const
   __shared__ double s_prof[3 * STRIDE_PROFILE_BINS];
   __shared__ int64_t s_tile;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  // launched as a programmatic dependent of the kernel that wrote the
+  // log-probs: wait for it (a no-op otherwise)
+  asm volatile("griddepcontrol.wait;" ::: "memory");
   if (tid == 0) s_tile = (int64_t)atomicAdd(p.ticket, 1u);
   if (tid < 3 * STRIDE_PROFILE_BINS) s_prof[tid] = 0.0;
   __syncthreads();
@@ -197,97 +202,88 @@ __global__ void __launch_bounds__(kScanTileRows) scan_logprobs_tile_kernel(const
   const int64_t t0 = tile * kScanTileRows;           // first window row of the tile
   const int64_t n_here = min((int64_t)kScanTileRows, p.n_rows - t0);
   const int64_t r0 = p.row_begin + t0;
-
-  // Layout checks, spread over every thread of the launch.
-  {
-    bool bad = false;
-    const int64_t stride = n_tiles * kScanTileRows;
-    for (int64_t k = t0 + tid; k < p.n_turns; k += stride)
-      bad |= __ldg(p.turn_row_off + k + 1) <= __ldg(p.turn_row_off + k);
-    for (int64_t i = t0 + tid; i < p.n_traj; i += stride) {
-      const int32_t a = __ldg(p.traj_turn_off + i), b = __ldg(p.traj_turn_off + i + 1);
-      if (a < 0 || b < a || b > p.n_turns) {
-        bad = true;
-      } else {
-        bad |= __ldg(p.turn_row_off + a) != __ldg(p.traj_row_off + i);
-        bad |= __ldg(p.turn_row_off + b) != __ldg(p.traj_row_off + i + 1);
-      }
-    }
-    if (bad) set_status(p.dev_status, STRIDE_DEV_BAD_LAYOUT);
+  const int64_t w = t0 + tid;  // this thread's window row
+  const int64_t r = p.row_begin + w;
+  const bool live = tid < n_here;
+  // the row's log-probs, in flight while the layout is looked up
+  float lps = 0.f, lpt = 0.f;
+  if (live) {
+    lps = __ldg(logp_s + w);
+    lpt = __ldg(logp_t + w);
   }
 
-  // 1. the tile's first turn and trajectory, then the staged offsets
+  // 1. the tile's first turn (warp 0) and first trajectory (warp 1), then
+  //    the offsets of the next kScanTileRows + 1 of each in shared memory
   if (warp == 0) {
-    const bool ok = p.n_turns > 0 && __ldg(p.turn_row_off) <= r0 && __ldg(p.traj_turn_off) <= 0;
-    int64_t k0 = 0, i0 = 0;
-    if (ok) {
-      k0 = warp_upper_le(p.turn_row_off, 0, p.n_turns - 1, r0, lane);
-      // trajectory holding turn k0: largest i with traj_turn_off[i] <= k0
-      int64_t lo = 0, hi = p.n_traj - 1;
-      while (hi > lo) {
-        const int64_t step = (hi - lo + 31) / 32;
-        const int64_t q = lo + step * (lane + 1);
-        const bool le = (q <= hi) && ((int64_t)__ldg(p.traj_turn_off + q) <= k0);
-        const int k = __popc(__ballot_sync(0xffffffffu, le));
-        const int64_t nlo = lo + step * k;
-        const int64_t nhi = (k < 32) ? min(hi, lo + step * (k + 1) - 1) : hi;
-        lo = nlo;
-        hi = nhi;
-      }
-      i0 = lo;
-    }
-    if (lane == 0) {
-      s_first[0] = ok ? k0 : -1;
-      s_first[1] = i0;
-    }
+    const bool ok = p.n_turns > 0 && __ldg(p.turn_row_off) <= r0;
+    const int64_t k0 = ok ? warp_upper_le(p.turn_row_off, 0, p.n_turns - 1, r0, lane) : 0;
+    if (lane == 0) s_first[0] = ok ? k0 : -1;
+  } else if (warp == 1) {
+    const bool ok = __ldg(p.traj_row_off) <= r0;
+    const int64_t i0 = ok ? warp_upper_le(p.traj_row_off, 0, p.n_traj - 1, r0, lane) : 0;
+    if (lane == 0) s_first[1] = ok ? i0 : -1;
   }
   __syncthreads();
   const int64_t k0 = s_first[0], i0 = s_first[1];
-  if (k0 >= 0) {
+  if (k0 >= 0 && i0 >= 0) {
     for (int j = tid; j <= kScanTileRows; j += kScanTileRows) {
       s_turn_off[j] = __ldg(p.turn_row_off + min(k0 + j, (int64_t)p.n_turns));
+      s_traj_row[j] = __ldg(p.traj_row_off + min(i0 + j, (int64_t)p.n_traj));
       s_traj_turn[j] = __ldg(p.traj_turn_off + min(i0 + j, (int64_t)p.n_traj));
     }
   }
   __syncthreads();
 
-  // 2. this thread's row and its element
-  const int64_t w = t0 + tid;  // window row
-  const int64_t r = p.row_begin + w;
-  const bool live = tid < n_here;
+  // 2. this thread's row: its turn and trajectory, and its element
   RowMeta meta;
   meta.bad = true;
   meta.traj = 0;
   meta.turn = 0;
   meta.local_turn = 0;
   meta.traj_start = meta.traj_end = meta.turn_start = meta.turn_end = 0;
-  if (live && k0 >= 0) {
+  if (live && k0 >= 0 && i0 >= 0) {
     const int nk = (int)min((int64_t)kScanTileRows, (int64_t)p.n_turns - k0);
     const int j = smem_upper_le(s_turn_off, nk, r);
-    const int64_t turn = k0 + j;
     const int ni = (int)min((int64_t)kScanTileRows, (int64_t)p.n_traj - i0);
-    const int q = smem_upper_le(s_traj_turn, ni, turn);
-    const int64_t traj = i0 + q;
+    int q = smem_upper_le(s_traj_row, ni, r);
+    int64_t traj = i0 + q, tr_start = s_traj_row[q], tr_end = s_traj_row[q + 1];
+    int64_t tu0 = s_traj_turn[q], tu1 = s_traj_turn[q + 1];
+    if (r >= tr_end && q == ni - 1 && i0 + ni < p.n_traj) {
+      // past the staged trajectories (more than kScanTileRows empty ones
+      // in the tile's rows): search the rest in global memory
+      int64_t lo = i0 + ni, hi = p.n_traj - 1;
+      while (lo < hi) {
+        const int64_t mid = (lo + hi + 1) >> 1;
+        if (__ldg(p.traj_row_off + mid) <= r) lo = mid; else hi = mid - 1;
+      }
+      traj = lo;
+      tr_start = __ldg(p.traj_row_off + traj);
+      tr_end = __ldg(p.traj_row_off + traj + 1);
+      tu0 = __ldg(p.traj_turn_off + traj);
+      tu1 = __ldg(p.traj_turn_off + traj + 1);
+    }
+    const int64_t turn = k0 + j;
     meta.turn = (int32_t)turn;
     meta.traj = (int32_t)traj;
     meta.turn_start = s_turn_off[j];
     meta.turn_end = s_turn_off[j + 1];
-    meta.local_turn = (int32_t)(turn - s_traj_turn[q]);
-    meta.traj_start = __ldg(p.traj_row_off + traj);
-    meta.traj_end = __ldg(p.traj_row_off + traj + 1);
-    meta.bad = !(meta.turn_start <= r && r < meta.turn_end) || !(meta.traj_start <= r && r < meta.traj_end) ||
-               !(s_traj_turn[q] <= turn && turn < s_traj_turn[q + 1]) || j + 1 > kScanTileRows;
+    meta.local_turn = (int32_t)(turn - tu0);
+    meta.traj_start = tr_start;
+    meta.traj_end = tr_end;
+    meta.bad = !(meta.turn_start <= r && r < meta.turn_end) || !(tr_start <= r && r < tr_end) ||
+               !(tu0 <= turn && turn < tu1);
   }
   TileElem x = {0.0, 0.0, 0.0, 0.0, 0};
   double c_before = 0.0, st_before = 0.0, e_sl = 0.0;
   int fturn = 0;
   if (live) {
     const float nan = __int_as_float(0x7fc00000);
-    float lps = __ldg(logp_s + w), lpt = __ldg(logp_t + w);
     if (meta.bad) {
       set_status(p.dev_status, STRIDE_DEV_BAD_LAYOUT);
       lps = nan;
       lpt = nan;
+      if (p.out.logp_s) p.out.logp_s[w] = nan;  // a bad row's log-probs are NaN
+      if (p.out.logp_t) p.out.logp_t[w] = nan;
     }
     const float dd = lps - lpt;
     if (p.out.opd) p.out.opd[w] = dd;
@@ -387,6 +383,25 @@ __global__ void __launch_bounds__(kScanTileRows) scan_logprobs_tile_kernel(const
     __syncthreads();
     if (tid < 3 * STRIDE_PROFILE_BINS && s_prof[tid] != 0.0) atomicAdd(p.profile + tid, s_prof[tid]);
   }
+
+  // Layout checks, spread over every thread of the launch (off the path of
+  // the scan: nothing above waits for them), unless the kernel that wrote
+  // the log-probs made them.
+  if (!validate) return;
+  bool bad = false;
+  const int64_t stride = n_tiles * kScanTileRows;
+  for (int64_t k = t0 + tid; k < p.n_turns; k += stride)
+    bad |= __ldg(p.turn_row_off + k + 1) <= __ldg(p.turn_row_off + k);
+  for (int64_t i = t0 + tid; i < p.n_traj; i += stride) {
+    const int32_t a = __ldg(p.traj_turn_off + i), b = __ldg(p.traj_turn_off + i + 1);
+    if (a < 0 || b < a || b > p.n_turns) {
+      bad = true;
+    } else {
+      bad |= __ldg(p.turn_row_off + a) != __ldg(p.traj_row_off + i);
+      bad |= __ldg(p.turn_row_off + b) != __ldg(p.traj_row_off + i + 1);
+    }
+  }
+  if (bad) set_status(p.dev_status, STRIDE_DEV_BAD_LAYOUT);
 }
 
 cudaError_t launch_partial_lse(const void* S, const void* T, int dtype, bool vec, int64_t ld,
@@ -417,9 +432,22 @@ cudaError_t launch_combine_partials(const float* parts, int32_t n_shards, int64_
 }
 
 cudaError_t launch_scan_logprobs(const BatchParams& p, const float* logp_s, const float* logp_t,
-                                 cudaStream_t stream) {
+                                 cudaStream_t stream, bool dependent) {
   const int64_t n_tiles = (p.n_rows + kScanTileRows - 1) / kScanTileRows;
-  scan_logprobs_tile_kernel<<<(unsigned)n_tiles, kScanTileRows, 0, stream>>>(p, logp_s, logp_t, n_tiles);
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)n_tiles);
+  cfg.blockDim = dim3(kScanTileRows);
+  cfg.dynamicSmemBytes = 0;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = dependent ? 1 : 0;
+  // the small-window kernel checks the layout itself (dependent launches)
+  const bool validate = !dependent;
+  const cudaError_t e = cudaLaunchKernelEx(&cfg, scan_logprobs_tile_kernel, p, logp_s, logp_t, n_tiles, validate);
+  if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }
 
