@@ -86,15 +86,12 @@ __global__ void __cluster_dims__(kStepCluster, 1, 1) __launch_bounds__(kStepThre
   const LT* srow = reinterpret_cast<const LT*>(p.S) + (int64_t)b * p.ld;
   const LT* trow = reinterpret_cast<const LT*>(p.T) + (int64_t)b * p.ld;
 
+  // The token id is loaded now and its logits gathered after the stream: a
+  // gather before it held rank 0 back by about 0.7 us on average (GB300
+  // timeline), and the cluster waits for its slowest rank.
   int32_t y = 0;
   float xs = nan, xt = nan;
-  if (rank == 0 && tid == 0) {
-    y = __ldg(p.tokens + b);
-    if (y >= 0 && y < p.V) {
-      xs = to_f32(srow[y]);
-      xt = to_f32(trow[y]);
-    }
-  }
+  if (rank == 0 && tid == 0) y = __ldg(p.tokens + b);
 
   // vocabulary slice of this rank (whole 16-byte vectors on the vector path;
   // the last rank also takes the ragged tail)
@@ -112,6 +109,10 @@ __global__ void __cluster_dims__(kStepCluster, 1, 1) __launch_bounds__(kStepThre
   }
   float mS = kMaxStart, sS = 0.f, mT = kMaxStart, sT = 0.f;
   stream_pair<LT, VEC, kStepUnroll>(srow, trow, c0, c1, tid, kStepThreads, mS, sS, mT, sT);
+  if (rank == 0 && tid == 0 && y >= 0 && y < p.V) {
+    xs = to_f32(srow[y]);
+    xt = to_f32(trow[y]);
+  }
   warp_merge2(mS, sS, mT, sT);
   if (lane == 0) {
     s_red[0][warp] = mS;

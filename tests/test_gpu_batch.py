@@ -81,7 +81,7 @@ LENS = [[1, 5, 17, 3], [9, 1], [33, 2, 1, 1, 4], [2]]
 
 
 @pytest.mark.parametrize("V,ld", [(151_936, 151_936), (151_933, 151_936), (151_933, 151_933),
-                                  (4099, 4099), (8, 8), (7, 8), (1, 1), (1, 8)])
+                                  (262_147, 262_152), (4099, 4099), (8, 8), (7, 8), (1, 1), (1, 8)])
 @pytest.mark.parametrize("mode", [0, 1])
 def test_bf16_ragged(stride, kernel, V, ld, mode):
     lay = synth.layout_from_turn_lengths(LENS)
