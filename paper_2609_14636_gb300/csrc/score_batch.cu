@@ -122,17 +122,12 @@ __global__ void __launch_bounds__(kSplitThreads, kSplitBlocksPerSm)
   const LT* srow = reinterpret_cast<const LT*>(p.S) + tile * p.ld;
   const LT* trow = teacher_row<LT>(p, tile);
 
+  // The token id is loaded now; its logits are gathered, and this row's
+  // share of the layout checks made (the scan skips them), after the
+  // stream, where they overlap the wait for the other ranks.
   int32_t y = 0;
   float xs = __int_as_float(0x7fc00000), xt = xs;
-  if (rank == 0 && tid == 0) {
-    y = __ldg(p.tokens + tile);
-    if (y >= 0 && y < p.V) {
-      xs = to_f32(srow[y]);
-      xt = to_f32(trow[y]);
-    }
-  } else if (rank == 0 && tid == 32) {
-    validate_layout(p, tile);  // this row's share of the layout checks (the scan skips them)
-  }
+  if (rank == 0 && tid == 0) y = __ldg(p.tokens + tile);
   int c0, c1;
   if (VEC) {
     constexpr int P = LogitTraits<LT>::kPerVec;
@@ -147,6 +142,12 @@ __global__ void __launch_bounds__(kSplitThreads, kSplitBlocksPerSm)
   }
   float mS = kMaxStart, sS = 0.f, mT = kMaxStart, sT = 0.f;
   stream_pair<LT, VEC, 4>(srow, trow, c0, c1, tid, kSplitThreads, mS, sS, mT, sT);
+  if (rank == 0 && tid == 0 && y >= 0 && y < p.V) {
+    xs = to_f32(srow[y]);
+    xt = to_f32(trow[y]);
+  } else if (rank == 0 && tid == 32) {
+    validate_layout(p, tile);
+  }
   warp_merge2(mS, sS, mT, sT);
   if (lane == 0) {
     s_red[0][warp] = mS;
