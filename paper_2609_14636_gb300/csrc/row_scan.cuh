@@ -315,10 +315,12 @@ __device__ __forceinline__ RowCarry row_finalize(const BatchParams& p, int64_t t
 // row_tail is the single-thread part once the row's inclusive prefix is
 // known: incl (running sum and open-turn sums through the row), c_before
 // and st_before (the running sum and open turn's sum of log pi_T before it);
-// of rc only rc.e.sl (the row's loss term) is read.
+// of rc only rc.e.sl (the row's loss term) is read.  With defer_traj the
+// trajectory's stop record and loss are left to the caller (the tiled scan
+// aggregates them per trajectory and tile).
 __device__ __forceinline__ void row_tail(const BatchParams& p, int64_t r, const RowMeta& meta,
                                          const RowCarry& rc, const ScanElem& incl, double c_before,
-                                         double st_before, bool timed_out);
+                                         double st_before, bool timed_out, bool defer_traj = false);
 
 __device__ __forceinline__ void row_resolve(const BatchParams& p, int64_t tile, int64_t r,
                                             const RowMeta& meta, RowCarry rc, int lane) {
@@ -341,7 +343,7 @@ __device__ __forceinline__ void row_resolve(const BatchParams& p, int64_t tile, 
 
 __device__ __forceinline__ void row_tail(const BatchParams& p, int64_t r, const RowMeta& meta,
                                          const RowCarry& rc, const ScanElem& incl, double c_before,
-                                         double st_before, bool timed_out) {
+                                         double st_before, bool timed_out, bool defer_traj) {
   if (timed_out) set_status(p.dev_status, STRIDE_DEV_TIMEOUT);
   if (meta.bad) return;
   const int64_t n_k = meta.turn_end - meta.turn_start;
@@ -361,16 +363,18 @@ __device__ __forceinline__ void row_tail(const BatchParams& p, int64_t r, const 
   const bool test = (p.mode == STRIDE_STOP_TOKEN_SUM) || turn_last;
   const float lam = p.lambda ? __ldg(p.lambda + meta.traj) : p.lambda_all;
   stride_scan_state* sp = p.state + meta.traj;
-  if (test && incl.c < (double)lam) {
-    atomicMin(reinterpret_cast<unsigned long long*>(&sp->stop_row),
-              (unsigned long long)(r - meta.traj_start));
-    atomicMin(reinterpret_cast<unsigned int*>(&sp->stop_turn), (unsigned int)meta.local_turn);
-    sp->stopped = 1;
-  }
-  const double before = (p.mode == STRIDE_STOP_TOKEN_SUM) ? c_before : c_before - st_before / (double)n_k;
-  if (before >= (double)lam) {
-    atomicAdd(&sp->loss, rc.e.sl);
-    atomicAdd(reinterpret_cast<unsigned long long*>(&sp->loss_tokens), 1ull);
+  if (!defer_traj) {
+    if (test && incl.c < (double)lam) {
+      atomicMin(reinterpret_cast<unsigned long long*>(&sp->stop_row),
+                (unsigned long long)(r - meta.traj_start));
+      atomicMin(reinterpret_cast<unsigned int*>(&sp->stop_turn), (unsigned int)meta.local_turn);
+      sp->stopped = 1;
+    }
+    const double before = (p.mode == STRIDE_STOP_TOKEN_SUM) ? c_before : c_before - st_before / (double)n_k;
+    if (before >= (double)lam) {
+      atomicAdd(&sp->loss, rc.e.sl);
+      atomicAdd(reinterpret_cast<unsigned long long*>(&sp->loss_tokens), 1ull);
+    }
   }
   if (r == meta.traj_end - 1 || r == p.row_end - 1) {
     sp->cum = incl.c;

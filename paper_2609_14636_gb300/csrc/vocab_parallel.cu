@@ -134,8 +134,12 @@ __global__ void combine_kernel(const float* __restrict__ parts, int32_t n_shards
 //      tile 0 always does), warp 0 folds its predecessors' (row_scan.cuh
 //      lookback) and publishes the tile's inclusive prefix;
 //   5. every row completes with its inclusive and exclusive prefixes: turn
-//      statistics, stop test, retained loss, carried state (row_tail), and
-//      the within-turn profile into the CTA's shared bins.
+//      statistics and carried state (row_tail), the within-turn profile into
+//      the CTA's shared bins;
+//   6. a second segmented scan (restarting at trajectory starts) gives each
+//      trajectory's retained loss and first crossing in the tile, so the
+//      trajectory's record takes one update per tile instead of one per row
+//      (the rows of a token-sum segment below lambda all contended for it).
 constexpr int kScanTileRows = 256;
 constexpr int kScanTileWarps = kScanTileRows / 32;
 constexpr int kRestartTurn = 1;  // st, sd, sl restart at this row
@@ -166,6 +170,67 @@ __device__ __forceinline__ TileElem tile_shfl_up(const TileElem& v, int d) {
   return o;
 }
 
+// Per-trajectory sums of the tile's rows for the trajectory's record: the
+// retained rows' loss terms and count, and whether a row crossed lambda.
+// Restarts at a trajectory's first row.
+struct TrajElem {
+  double loss;
+  int count;
+  int crossed;
+  int restart;
+};
+
+__device__ __forceinline__ TrajElem traj_combine(const TrajElem& a, const TrajElem& b) {
+  if (b.restart) return b;
+  return TrajElem{a.loss + b.loss, a.count + b.count, a.crossed | b.crossed, a.restart};
+}
+
+__device__ __forceinline__ TrajElem traj_shfl_up(const TrajElem& v, int d) {
+  TrajElem o;
+  o.loss = __shfl_up_sync(0xffffffffu, v.loss, d);
+  o.count = __shfl_up_sync(0xffffffffu, v.count, d);
+  o.crossed = __shfl_up_sync(0xffffffffu, v.crossed, d);
+  o.restart = __shfl_up_sync(0xffffffffu, v.restart, d);
+  return o;
+}
+
+__device__ __forceinline__ TileElem elem_combine(const TileElem& a, const TileElem& b) { return tile_combine(a, b); }
+__device__ __forceinline__ TrajElem elem_combine(const TrajElem& a, const TrajElem& b) { return traj_combine(a, b); }
+__device__ __forceinline__ TileElem elem_shfl_up(const TileElem& v, int d) { return tile_shfl_up(v, d); }
+__device__ __forceinline__ TrajElem elem_shfl_up(const TrajElem& v, int d) { return traj_shfl_up(v, d); }
+
+// Inclusive and exclusive scan of one element per thread over the CTA's
+// kScanTileRows threads, in thread order: warp shuffles, then warp 0 scans
+// the warps' totals once (each thread then combines with one prefix).
+// `id` is the identity; s_tot and s_pre hold kScanTileWarps elements.
+template <typename E>
+__device__ __forceinline__ void block_scan(const E& v, const E& id, int lane, int warp, E* s_tot, E* s_pre,
+                                           E& incl_out, E& excl_out) {
+  E incl = v;
+#pragma unroll
+  for (int d = 1; d < 32; d <<= 1) {
+    const E o = elem_shfl_up(incl, d);
+    if (lane >= d) incl = elem_combine(o, incl);
+  }
+  const E up1 = elem_shfl_up(incl, 1);
+  if (lane == 31) s_tot[warp] = incl;
+  __syncthreads();
+  if (warp == 0) {
+    E t = lane < kScanTileWarps ? s_tot[lane] : id;
+#pragma unroll
+    for (int d = 1; d < kScanTileWarps; d <<= 1) {
+      const E o = elem_shfl_up(t, d);
+      if (lane >= d) t = elem_combine(o, t);
+    }
+    const E e = elem_shfl_up(t, 1);
+    if (lane < kScanTileWarps) s_pre[lane] = (lane == 0) ? id : e;
+  }
+  __syncthreads();
+  const E wpre = s_pre[warp];
+  incl_out = elem_combine(wpre, incl);
+  excl_out = (lane == 0) ? wpre : elem_combine(wpre, up1);
+}
+
 // Largest j in [0, n) with a[j] <= r (a ascending, a[0] <= r).
 __device__ __forceinline__ int smem_upper_le(const int64_t* a, int n, int64_t r) {
   int lo = 0, hi = n - 1;
@@ -185,6 +250,9 @@ __global__ void __launch_bounds__(kScanTileRows) scan_logprobs_tile_kernel(const
   __shared__ int64_t s_traj_turn[kScanTileRows + 1];  // traj_turn_off, widened
   __shared__ int64_t s_first[2];                      // first turn, first trajectory of the tile
   __shared__ TileElem s_wtot[kScanTileWarps];
+  __shared__ TileElem s_wpre[kScanTileWarps];
+  __shared__ TrajElem s_ttot[kScanTileWarps];
+  __shared__ TrajElem s_tpre[kScanTileWarps];
   __shared__ TileElem s_excl;
   __shared__ TileElem s_agg;
   __shared__ int s_flags;  // bit 0: lookback timed out
@@ -274,7 +342,7 @@ __global__ void __launch_bounds__(kScanTileRows) scan_logprobs_tile_kernel(const
                !(tu0 <= turn && turn < tu1);
   }
   TileElem x = {0.0, 0.0, 0.0, 0.0, 0};
-  double c_before = 0.0, st_before = 0.0, e_sl = 0.0;
+  double c_before = 0.0, st_before = 0.0, e_sl = 0.0, ri_c = 0.0;
   int fturn = 0;
   if (live) {
     const float nan = __int_as_float(0x7fc00000);
@@ -317,19 +385,9 @@ __global__ void __launch_bounds__(kScanTileRows) scan_logprobs_tile_kernel(const
   }
 
   // 3. segmented inclusive scan over the tile
-  TileElem incl = x;
-#pragma unroll
-  for (int d = 1; d < 32; d <<= 1) {
-    const TileElem o = tile_shfl_up(incl, d);
-    if (lane >= d) incl = tile_combine(o, incl);
-  }
-  TileElem excl_in_warp = tile_shfl_up(incl, 1);
-  if (lane == 31) s_wtot[warp] = incl;
-  __syncthreads();
-  TileElem wpre = {0.0, 0.0, 0.0, 0.0, 0};
-  for (int v = 0; v < warp; ++v) wpre = tile_combine(wpre, s_wtot[v]);
-  const TileElem tile_incl = tile_combine(wpre, incl);
-  const TileElem tile_excl = (lane == 0) ? wpre : tile_combine(wpre, excl_in_warp);
+  const TileElem tile_id = {0.0, 0.0, 0.0, 0.0, 0};
+  TileElem tile_incl, tile_excl;
+  block_scan(x, tile_id, lane, warp, s_wtot, s_wpre, tile_incl, tile_excl);
 
   // 4. publish the tile's aggregate, fold predecessors, publish its prefix
   if (tid == (int)(n_here - 1)) {
@@ -377,7 +435,41 @@ __global__ void __launch_bounds__(kScanTileRows) scan_logprobs_tile_kernel(const
     RowCarry rc;
     rc.e = ScanElem{0.0, 0.0, 0.0, e_sl, fturn};
     const ScanElem si{ri.c, ri.st, ri.sd, ri.sl, 1};
-    row_tail(p, r, meta, rc, si, c_before, st_before, (s_flags & 1) != 0);
+    row_tail(p, r, meta, rc, si, c_before, st_before, (s_flags & 1) != 0, true);
+    ri_c = ri.c;
+  }
+
+  // 6. the trajectories' stop records and losses, once per trajectory and
+  //    tile: the first row of a trajectory here that crosses lambda records
+  //    the stop (the running sum never rises, so it is the trajectory's
+  //    first crossing unless an earlier tile's is lower), and the last row
+  //    of a trajectory here adds its retained rows' loss and count.
+  TrajElem te = {0.0, 0, 0, 1};
+  bool cross = false;
+  if (live && !meta.bad) {
+    const int64_t n_k = meta.turn_end - meta.turn_start;
+    const bool turn_last = (r == meta.turn_end - 1);
+    const bool test = (p.mode == STRIDE_STOP_TOKEN_SUM) || turn_last;
+    const float lam = p.lambda ? __ldg(p.lambda + meta.traj) : p.lambda_all;
+    cross = test && ri_c < (double)lam;
+    const double before = (p.mode == STRIDE_STOP_TOKEN_SUM) ? c_before : c_before - st_before / (double)n_k;
+    const bool kept = before >= (double)lam;
+    te = TrajElem{kept ? e_sl : 0.0, kept ? 1 : 0, cross ? 1 : 0, r == meta.traj_start ? 1 : 0};
+  }
+  const TrajElem traj_id = {0.0, 0, 0, 0};
+  TrajElem t_incl, t_excl;
+  block_scan(te, traj_id, lane, warp, s_ttot, s_tpre, t_incl, t_excl);
+  if (live && !meta.bad) {
+    stride_scan_state* sp = p.state + meta.traj;
+    if (cross && (te.restart || !t_excl.crossed)) {
+      atomicMin(reinterpret_cast<unsigned long long*>(&sp->stop_row), (unsigned long long)(r - meta.traj_start));
+      atomicMin(reinterpret_cast<unsigned int*>(&sp->stop_turn), (unsigned int)meta.local_turn);
+      sp->stopped = 1;
+    }
+    if ((r == meta.traj_end - 1 || tid == (int)(n_here - 1)) && t_incl.count > 0) {
+      atomicAdd(&sp->loss, t_incl.loss);
+      atomicAdd(reinterpret_cast<unsigned long long*>(&sp->loss_tokens), (unsigned long long)t_incl.count);
+    }
   }
   if (p.profile) {
     __syncthreads();
