@@ -806,12 +806,14 @@ def run_tiny(args) -> None:
             "roofline": {"bound": "hbm", "achieved": bpr * R / (ms * 1e-3) / 1e9, "peak": peak, "unit": "GB/s",
                          "frac": bpr * R / (ms * 1e-3) / 1e9 / peak, "traffic": None,
                          "algorithmic_bytes_per_launch": bpr * R,
-                         "kernel": "score_batch_split_kernel<f32> (2-CTA clusters, one wave of 1,024 CTAs)",
+                         "kernel": "score_batch_split_kernel<f32> (2-CTA clusters, one wave of 1,024 CTAs) "
+                                   "+ scan_logprobs_tile_kernel (2 tiles of 256 rows)",
                          "note": "512 rows on 152 SMs: a latency-bound launch; time includes state init"},
             "cpu_baseline": {"value": cpu_rate, "unit": UNIT, "cores": threads, "kind": "oracle",
                              "sample": f"all {R} rows"},
-            "clocks": clk.summary(), "gpu_launches": 2 * args.steps,
-            "graph": "state init + workspace clear + scoring, one CUDA graph replayed per step",
+            "clocks": clk.summary(), "gpu_launches": 3 * args.steps,
+            "graph": "state init + workspace clear + small-window scoring + tiled scan, one CUDA graph "
+                     "replayed per step",
         })
         print(json.dumps(line), flush=True)
 
