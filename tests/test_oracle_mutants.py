@@ -48,6 +48,9 @@ MUTANTS = [
     ("record_drops_prefix", "int32_t len = keep;", "int32_t len = 0;"),
     ("record_no_clamp", "if (keep > n_turns[x]) keep = n_turns[x];", "if (keep > T_max) keep = T_max;"),
     ("record_prefix_off_by_one", "int32_t keep = k0 ? k0[i] : 0;", "int32_t keep = k0 ? k0[i] + 1 : 0;"),
+    ("f32_logit_ignores_row", "    return (double)p[r * ld + j];", "    return (double)p[j];"),
+    ("thread_split_drops_row", "jb->r1 = rows * (i + 1) / nthreads;",
+     "jb->r1 = rows * (i + 1) / nthreads - (i + 1 < nthreads ? 1 : 0);"),
 ]
 
 
