@@ -20,12 +20,35 @@
 #include <stdlib.h>
 #include <string.h>
 
+#include <atomic>
+
 #include "stride.h"
 #include "stride_device.cuh"
 #include "stride_internal.h"
 #include "row_scan.cuh"
 
 namespace stride {
+
+int current_device_sms(int* dev_out, cudaError_t* err) {
+  constexpr int kMaxDev = 64;
+  static std::atomic<int> cache[kMaxDev];  // 0 = not looked up yet
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (dev_out) *dev_out = dev;
+  if (e != cudaSuccess || dev < 0 || dev >= kMaxDev) {
+    if (err) *err = e != cudaSuccess ? e : cudaErrorInvalidDevice;
+    return 0;
+  }
+  int sms = cache[dev].load(std::memory_order_relaxed);
+  if (sms > 0) return sms;
+  e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  if (e != cudaSuccess || sms <= 0) {
+    if (err) *err = e != cudaSuccess ? e : cudaErrorInvalidDevice;
+    return 0;
+  }
+  cache[dev].store(sms, std::memory_order_relaxed);
+  return sms;
+}
 
 constexpr int kBatchThreads = 512;
 constexpr int kBatchWarps = kBatchThreads / 32;
@@ -292,11 +315,10 @@ cudaError_t launch_score_batch(const BatchParams& p, int dtype, bool vec, cudaSt
   // aligned rows with at least one whole vector otherwise take the
   // persistent bulk-copy kernel (score_batch_stream.cu); the rest take one
   // CTA per row.
-  static int sm_count[64] = {0};
   int dev = 0;
-  if (cudaGetDevice(&dev) == cudaSuccess && dev >= 0 && dev < 64 && sm_count[dev] == 0)
-    cudaDeviceGetAttribute(&sm_count[dev], cudaDevAttrMultiProcessorCount, dev);
-  const int sms = (dev >= 0 && dev < 64 && sm_count[dev] > 0) ? sm_count[dev] : 152;
+  cudaError_t qe = cudaSuccess;
+  const int sms = current_device_sms(&dev, &qe);
+  if (sms <= 0) return qe != cudaSuccess ? qe : cudaErrorInvalidDevice;
   // STRIDE_BATCH_KERNEL = split | split1 | split2 | split4 | split8 |
   // stream | rows forces one kernel, or the split kernel with one cluster
   // size (tests and diagnosis); anything else, or unset, chooses by window

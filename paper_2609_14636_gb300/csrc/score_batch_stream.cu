@@ -36,6 +36,8 @@
 // issuing, waits (bounded) for the copies it has in flight, and returns.
 #include <math.h>
 
+#include <atomic>
+
 #include "mbarrier.cuh"
 #include "row_scan.cuh"
 #include "stride.h"
@@ -381,27 +383,25 @@ __global__ void __launch_bounds__(kStreamThreads, 1) score_batch_stream_kernel(c
 size_t stream_smem_bytes() { return kStreamSmem; }
 
 cudaError_t launch_score_batch_stream(const BatchParams& p, int dtype, cudaStream_t stream) {
-  static int sm_count[64] = {0};
-  static bool attr_done[2] = {false, false};
+  // The dynamic shared-memory limit is a per-device function attribute: set
+  // once per device and dtype (setting it again is harmless, so two threads
+  // racing here both succeed).
+  static std::atomic<bool> attr_done[64][2];
   int dev = 0;
-  cudaError_t e = cudaGetDevice(&dev);
-  if (e != cudaSuccess) return e;
-  if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
-  if (sm_count[dev] == 0) {
-    e = cudaDeviceGetAttribute(&sm_count[dev], cudaDevAttrMultiProcessorCount, dev);
-    if (e != cudaSuccess) return e;
-  }
+  cudaError_t e = cudaSuccess;
+  const int sms = current_device_sms(&dev, &e);
+  if (sms <= 0) return e != cudaSuccess ? e : cudaErrorInvalidDevice;
   const int di = dtype == STRIDE_DTYPE_BF16 ? 0 : 1;
-  if (!attr_done[di]) {
+  if (!attr_done[dev][di].load(std::memory_order_acquire)) {
     e = dtype == STRIDE_DTYPE_BF16
             ? cudaFuncSetAttribute(score_batch_stream_kernel<__nv_bfloat16>,
                                    cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kStreamSmem)
             : cudaFuncSetAttribute(score_batch_stream_kernel<float>,
                                    cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kStreamSmem);
     if (e != cudaSuccess) return e;
-    attr_done[di] = true;
+    attr_done[dev][di].store(true, std::memory_order_release);
   }
-  const int64_t grid = p.n_rows < sm_count[dev] ? p.n_rows : sm_count[dev];
+  const int64_t grid = p.n_rows < sms ? p.n_rows : sms;
   if (dtype == STRIDE_DTYPE_BF16)
     score_batch_stream_kernel<__nv_bfloat16><<<(unsigned)grid, kStreamThreads, kStreamSmem, stream>>>(p);
   else

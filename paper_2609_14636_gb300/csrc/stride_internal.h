@@ -108,6 +108,10 @@ struct TeacherTable {
 cudaError_t launch_teacher_rows(const BatchParams& p, const TeacherTable& tt, const uint8_t* traj_domain,
                                 const int64_t* traj_T_row0, const void** rows_out, cudaStream_t stream);
 
+// Multiprocessor count of the current device, looked up once per device
+// (thread-safe); 0 with the CUDA error in *err if it cannot be queried.
+int current_device_sms(int* dev_out, cudaError_t* err);
+
 // Launchers return a cudaError_t from the launch.
 cudaError_t launch_score_batch(const BatchParams& p, int dtype, bool vec, cudaStream_t stream);
 cudaError_t launch_score_batch_stream(const BatchParams& p, int dtype, cudaStream_t stream);
