@@ -45,9 +45,10 @@
  * - Turn and row indices reported per trajectory are 0-based and local to the
  *   trajectory.  The paper's turns are 1-based, so the returned k* equals its
  *   K0 = k* - 1 (Algorithm 1): the number of turns reused as context.
- * - Every compute call is a plain kernel launch (plus cudaMemsetAsync of the
- *   workspace for stride_score_batch), so a sequence of calls can be captured
- *   in a CUDA graph.
+ * - Every compute call is a plain kernel launch or two (plus a
+ *   cudaMemsetAsync of the workspace on the batch paths other than the
+ *   small-window one), so a sequence of calls can be captured in a CUDA
+ *   graph.
  * - The library is built for sm_103a only; on another device the calls return
  *   STRIDE_ERR_UNSUPPORTED_DEVICE.  There is no CPU fallback.
  * - The batch calls choose among three kernels with the same results: for

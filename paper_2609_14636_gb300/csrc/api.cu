@@ -175,9 +175,9 @@ int stride_score_batch(const void* S, const void* T, int32_t dtype, int64_t ld, 
                                workspace_bytes, 0);
   if (rc != STRIDE_OK || row_end == row_begin) return rc;
   cudaStream_t st = (cudaStream_t)stream;
-  if (cudaMemsetAsync(workspace, 0, L.clear_bytes, st) != cudaSuccess) return STRIDE_ERR_CUDA;
   const bool vec = vector_ok(S, T, dtype, ld);
-  return stride::launch_score_batch(p, dtype, vec, st) == cudaSuccess ? STRIDE_OK : STRIDE_ERR_CUDA;
+  return stride::launch_score_batch(p, dtype, vec, L.clear_bytes, st) == cudaSuccess ? STRIDE_OK
+                                                                                     : STRIDE_ERR_CUDA;
 }
 
 int stride_score_batch_multi_teacher(const void* S, const void* const* T_domains,
@@ -215,13 +215,13 @@ int stride_score_batch_multi_teacher(const void* S, const void* const* T_domains
   if (rc != STRIDE_OK || n_rows == 0) return rc;
   const void** rows = reinterpret_cast<const void**>(static_cast<char*>(workspace) + L.total);
   cudaStream_t st = (cudaStream_t)stream;
-  if (cudaMemsetAsync(workspace, 0, L.clear_bytes, st) != cudaSuccess) return STRIDE_ERR_CUDA;
   if (stride::launch_teacher_rows(p, tt, traj_domain, traj_T_row0, rows, st) != cudaSuccess)
     return STRIDE_ERR_CUDA;
   p.T_rows = rows;
   const bool vec = aligned && aligned16(S) && ((ld * (int64_t)dtype_bytes(dtype)) % 16) == 0 &&
                    (tt.ld_bytes % 16) == 0;
-  return stride::launch_score_batch(p, dtype, vec, st) == cudaSuccess ? STRIDE_OK : STRIDE_ERR_CUDA;
+  return stride::launch_score_batch(p, dtype, vec, L.clear_bytes, st) == cudaSuccess ? STRIDE_OK
+                                                                                     : STRIDE_ERR_CUDA;
 }
 
 int stride_score_step(const void* S, const void* T, int32_t dtype, int64_t ld, int64_t V,

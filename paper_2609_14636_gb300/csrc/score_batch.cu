@@ -137,6 +137,14 @@ __global__ void __launch_bounds__(kSplitThreads, kSplitBlocksPerSm)
   __shared__ float s_part[4];
   // the dependent scan may be scheduled once every CTA of this grid runs
   asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+  if (blockIdx.x == 0) {
+    // What the scan needs at zero: its tile ticket (the header's second
+    // word) and one flag per 256-row tile.  The scan reads them only after
+    // this grid has completed.
+    const int64_t n_tiles = (p.n_rows + 255) / 256;
+    for (int64_t t = threadIdx.x; t < n_tiles; t += blockDim.x) p.flags[t * kFlagStride] = 0u;
+    if (threadIdx.x == 0) p.ticket[1] = 0u;
+  }
   cg::cluster_group cluster = cg::this_cluster();
   const int rank = (int)cluster.block_rank();
   const int n_ranks = (int)cluster.num_blocks();
@@ -310,7 +318,7 @@ static cudaError_t launch_split(const BatchParams& p, int C, cudaStream_t stream
   return cudaLaunchKernelEx(&cfg, score_batch_split_kernel<LT, VEC>, p);
 }
 
-cudaError_t launch_score_batch(const BatchParams& p, int dtype, bool vec, cudaStream_t stream) {
+cudaError_t launch_score_batch(const BatchParams& p, int dtype, bool vec, size_t clear_bytes, cudaStream_t stream) {
   // Small windows split each row over a cluster (split_cluster); 16-byte-
   // aligned rows with at least one whole vector otherwise take the
   // persistent bulk-copy kernel (score_batch_stream.cu); the rest take one
@@ -335,6 +343,7 @@ cudaError_t launch_score_batch(const BatchParams& p, int dtype, bool vec, cudaSt
   }
   if (C > 0 && p.V < 32 * (int64_t)C) C = f_split ? 1 : 0;  // a few logits per rank at least
   if (C > 0) {
+    // no memset: the split kernel clears the scan's ticket and tile flags
     cudaError_t e;
     if (dtype == STRIDE_DTYPE_BF16)
       e = vec ? launch_split<__nv_bfloat16, true>(p, C, stream) : launch_split<__nv_bfloat16, false>(p, C, stream);
@@ -346,6 +355,10 @@ cudaError_t launch_score_batch(const BatchParams& p, int dtype, bool vec, cudaSt
     BatchParams q = p;
     q.ticket = p.ticket + 1;
     return launch_scan_logprobs(q, p.ws_logp_s, p.ws_logp_t, stream, true);
+  }
+  {
+    const cudaError_t e = cudaMemsetAsync(p.ticket, 0, clear_bytes, stream);
+    if (e != cudaSuccess) return e;
   }
   const int per_vec = dtype == STRIDE_DTYPE_BF16 ? 8 : 4;
   if (vec && p.V >= per_vec && !f_rows) return launch_score_batch_stream(p, dtype, stream);

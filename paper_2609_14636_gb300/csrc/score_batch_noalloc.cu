@@ -16,9 +16,10 @@
 //   STRIDE_ERR_TOO_LARGE before anything is launched);
 // - every call, on every stream, shares the one array per device, and the
 //   array keeps the previous call's contents: the call clears the part that
-//   must start at zero (ticket and row flags) with cudaMemsetAsync before its
-//   kernel.  Two calls that overlap in time on the GPU race on the array and
-//   give wrong results: order them on one stream (or with events);
+//   must start at zero (tickets and flags) before its scan reads it (with
+//   cudaMemsetAsync, or from the small-window kernel).  Two calls that
+//   overlap in time on the GPU race on the array and give wrong results:
+//   order them on one stream (or with events);
 // - the first call on a device looks up the array's device address with
 //   cudaGetSymbolAddress (this may load the library's module onto the
 //   device); make that first call before any stream capture.
@@ -86,8 +87,8 @@ extern "C" STRIDE_API int stride_score_batch_noalloc(
   void* scratch = nullptr;
   const int sc = scratch_for_current_device(&scratch);
   if (sc != STRIDE_OK) return sc;
-  // The scoring entry point clears the ticket and flags of the window and
-  // launches the kernel with pointers into the scratch.
+  // The scoring entry point clears the tickets and flags of the window and
+  // launches the kernels with pointers into the scratch.
   return stride_score_batch(S, T, dtype, ld, V, tokens, traj_row_off, turn_row_off, traj_turn_off,
                             n_traj, n_turns, row_begin, row_end, stop_mode, lambda, lambda_all,
                             state, out, turn_stats, profile, dev_status, scratch, kNoAllocBytes,

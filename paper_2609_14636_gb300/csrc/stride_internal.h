@@ -113,7 +113,10 @@ cudaError_t launch_teacher_rows(const BatchParams& p, const TeacherTable& tt, co
 int current_device_sms(int* dev_out, cudaError_t* err);
 
 // Launchers return a cudaError_t from the launch.
-cudaError_t launch_score_batch(const BatchParams& p, int dtype, bool vec, cudaStream_t stream);
+// Clears what must start at zero in the workspace (clear_bytes from its
+// start: a memset, or on the small-window path the kernel itself) and
+// launches the batch scoring kernels.
+cudaError_t launch_score_batch(const BatchParams& p, int dtype, bool vec, size_t clear_bytes, cudaStream_t stream);
 cudaError_t launch_score_batch_stream(const BatchParams& p, int dtype, cudaStream_t stream);
 cudaError_t launch_score_step(const StepParams& p, int dtype, bool vec, cudaStream_t stream);
 cudaError_t launch_select_restart(const SelectParams& p, cudaStream_t stream);
