@@ -374,6 +374,21 @@ def run_batch(args) -> None:
     ms_step = ms_total / args.steps
     value = whole_job_rate(R, ws, ms_step)
 
+    # the same scoring calls with the within-turn profile (Observation 1)
+    # accumulated too, outside the timed steps above
+    prof = stride.new_profile(dev)
+    pev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(5)]
+    for a, b in pev:
+        stride.stride_state_init(st, lay.n_traj, stream)
+        a.record(stream)
+        for wa, wb in windows:
+            stride.stride_score_batch(S[wa:wb], T[wa:wb], tok[wa:wb], *offs, wa, wb, stride.TURN_MEAN, lam_d, st,
+                                      out={k: v[wa:wb] for k, v in out.items()}, turn_stats=ts,
+                                      dev_status=status, workspace=wsb, stream=stream, profile=prof)
+        b.record(stream)
+    torch.cuda.synchronize()
+    ms_with_profile = statistics.mean(a.elapsed_time(b) for a, b in pev)
+
     # ---- roofline of the fused kernel -------------------------------------
     peaks = measured_peaks()
     peak = peaks.get("hbm_gbs", 6800.0)
@@ -385,6 +400,7 @@ def run_batch(args) -> None:
                 "traffic": None if dram_per_row is None else dram_per_row * R,
                 "algorithmic_bytes_per_launch": bpr * R, "kernel_ms_mean": k_avg,
                 "kernel_ms_min": min(k_ms), "kernel": "score_batch_stream_kernel<bf16>",
+                "kernel_ms_mean_with_profile": ms_with_profile,
                 "peak_source": "MEASURED_PEAKS.json hbm_gbs (of measured)" if "hbm_gbs" in peaks else "fallback 6.8 TB/s"}
 
     # ---- end to end from pinned host buffers ------------------------------
@@ -726,6 +742,30 @@ def run_select(args) -> None:
     us_call = 1e3 * a.elapsed_time(b) / (reps * calls)
     us_call = max_over_ranks(us_call, dev)
     bytes_call = N * T_max * 5 + N * 12
+
+    # the prefix buffer's record step (Algorithm 1): 128 rollouts of 12 turns
+    # each recorded into a copy of the buffer, each keeping k0 stored turns
+    n_rec, turns_rec = 128, 12
+    rng = np.random.default_rng(9)
+    rbuf, rnt = means.clone(), nt.clone()
+    tasks = torch.from_numpy(rng.choice(N, n_rec, replace=False).astype(np.int32)).to(dev)
+    k0 = torch.from_numpy(rng.integers(0, 6, n_rec).astype(np.int32)).to(dev)
+    rts = stride.new_turn_stats(n_rec * turns_rec, dev)
+    rts_view = rts.view(-1, stride.TURN_STATS_DTYPE.itemsize)
+    tt = np.zeros(n_rec * turns_rec, stride.TURN_STATS_DTYPE)
+    tt["mean_t"] = rng.normal(-4.5, 1.5, n_rec * turns_rec).astype(np.float32)
+    tt["n"] = 100
+    rts_view.copy_(torch.from_numpy(tt.view(np.uint8).reshape(n_rec * turns_rec, -1)).to(dev))
+    rturn_off = torch.arange(0, n_rec * turns_rec + 1, turns_rec, dtype=torch.int32, device=dev)
+    g_rec = _graph(lambda: [stride.stride_buffer_record(rbuf, rnt, tasks, k0, rts, rturn_off) for _ in range(calls)])
+    for _ in range(3):
+        g_rec.replay()
+    a.record(stream)
+    for _ in range(reps):
+        g_rec.replay()
+    b.record(stream)
+    torch.cuda.synchronize()
+    us_record = 1e3 * a.elapsed_time(b) / (reps * calls)
     if rank == 0:
         line = _common_line(args, ws, us_call / 1e3, ws * N / (us_call * 1e-6), unit="records/s",
                             metric="restart choices/sec (10,000 x 12 records)", dtype="f32")
@@ -734,8 +774,11 @@ def run_select(args) -> None:
                        "mask": "Bernoulli(0.5)", "alpha": -6.0, "graph": f"{calls} launches per CUDA graph"},
             "roofline": {"bound": "latency", "achieved": bytes_call / (us_call * 1e-6) / 1e9, "peak": None,
                          "unit": "GB/s", "frac": None, "traffic": None, "us_per_call": us_call,
-                         "kernel": "select_restart_kernel (one warp per record)"},
-            "clocks": clk.summary(), "gpu_launches": reps * calls,
+                         "kernel": "select_restart_kernel (one warp per record)",
+                         "record_us_per_call": us_record,
+                         "record": f"stride_buffer_record of {n_rec} rollouts x {turns_rec} turns into the "
+                                   f"{N}-record buffer (buffer_record_kernel, {calls} launches per graph)"},
+            "clocks": clk.summary(), "gpu_launches": 2 * reps * calls,
         })
         print(json.dumps(line), flush=True)
 
