@@ -188,9 +188,51 @@ __device__ __forceinline__ void stream_pair(const LT* __restrict__ srow, const L
       lse_one(to_f32(trow[j]), mT, sT);
     }
   } else {
-    for (int j = c0 + tid; j < c1; j += nthreads) {
+    // Rows that are not 16-byte aligned.  When S and T share the row's
+    // misalignment (row stride and bases alike), the logits up to the next
+    // 16-byte boundary are read one by one and the rest as 16-byte vectors,
+    // then the ragged tail; otherwise every logit is read on its own.
+    // (A typed pointer is element-aligned, so the distance to the boundary
+    // is a whole number of elements.)
+    const uintptr_t as = reinterpret_cast<uintptr_t>(srow + c0), at = reinterpret_cast<uintptr_t>(trow + c0);
+    const bool same = ((as ^ at) & 15u) == 0;
+    int head = c1 - c0;
+    if (same) {
+      const int h = (int)(((16u - (unsigned)(as & 15u)) & 15u) / sizeof(LT));
+      head = h < head ? h : head;
+    }
+    for (int j = c0 + tid; j < c0 + head; j += nthreads) {
       lse_one(to_f32(srow[j]), mS, sS);
       lse_one(to_f32(trow[j]), mT, sT);
+    }
+    if (same && c0 + head < c1) {
+      const LT* s2 = srow + c0 + head;  // 16-byte aligned
+      const LT* t2 = trow + c0 + head;
+      const int n2 = c1 - (c0 + head);
+      const int nvec = n2 / P;
+      const uint4* sv = reinterpret_cast<const uint4*>(s2);
+      const uint4* tv = reinterpret_cast<const uint4*>(t2);
+      int v = tid;
+      for (; v + (U - 1) * nthreads < nvec; v += U * nthreads) {
+        uint4 a[U], b[U];
+#pragma unroll
+        for (int u = 0; u < U; ++u) {
+          a[u] = ld_stream(sv + v + u * nthreads);
+          b[u] = ld_stream(tv + v + u * nthreads);
+        }
+        LogitTraits<LT>::template chunk<U>(a, mS, sS);
+        LogitTraits<LT>::template chunk<U>(b, mT, sT);
+      }
+      for (; v < nvec; v += nthreads) {
+        uint4 a[1] = {ld_stream(sv + v)};
+        uint4 b[1] = {ld_stream(tv + v)};
+        LogitTraits<LT>::template chunk<1>(a, mS, sS);
+        LogitTraits<LT>::template chunk<1>(b, mT, sT);
+      }
+      for (int j = nvec * P + tid; j < n2; j += nthreads) {
+        lse_one(to_f32(s2[j]), mS, sS);
+        lse_one(to_f32(t2[j]), mT, sT);
+      }
     }
   }
 }
