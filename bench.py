@@ -39,7 +39,7 @@ import numpy as np
 ROOT = Path(__file__).resolve().parent
 sys.path.insert(0, str(ROOT))
 
-METRIC = "scored tokens/sec (V=151,936 bf16)"
+METRIC = "scored tokens/sec and achieved HBM GB/s (% of GB300 peak) at V=151,936 bf16"  # value: tokens/s; GB/s and its fraction: roofline
 UNIT = "tokens/s"
 
 
