@@ -855,7 +855,7 @@ def run_tiny(args) -> None:
             "cpu_baseline": {"value": cpu_rate, "unit": UNIT, "cores": threads, "kind": "oracle",
                              "sample": f"all {R} rows"},
             "clocks": clk.summary(), "gpu_launches": 3 * args.steps,
-            "graph": "state init + workspace clear + small-window scoring + tiled scan, one CUDA graph "
+            "graph": "state init + small-window scoring + tiled scan, one CUDA graph "
                      "replayed per step",
         })
         print(json.dumps(line), flush=True)

@@ -135,7 +135,13 @@ __global__ void __launch_bounds__(kSplitThreads, kSplitBlocksPerSm)
     score_batch_split_kernel(const BatchParams p) {
   __shared__ float s_red[4][kSplitWarps];
   __shared__ float s_part[4];
-  // the dependent scan may be scheduled once every CTA of this grid runs
+  // Launched as a programmatic dependent of the previous kernel on the
+  // stream: the CTAs may be scheduled while it finishes, and each waits for
+  // its completion before the first global access.  Only then may the
+  // dependent scan be scheduled, so that whatever the previous kernels
+  // wrote (the layout, the carried state) is complete when the scan reads
+  // it before its own wait.
+  asm volatile("griddepcontrol.wait;" ::: "memory");
   asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
   if (blockIdx.x == 0) {
     // What the scan needs at zero: its tile ticket (the header's second
@@ -308,13 +314,15 @@ static cudaError_t launch_split(const BatchParams& p, int C, cudaStream_t stream
   cfg.blockDim = dim3(kSplitThreads);
   cfg.dynamicSmemBytes = 0;
   cfg.stream = stream;
-  cudaLaunchAttribute attr[1];
+  cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeClusterDimension;
   attr[0].val.clusterDim.x = (unsigned)C;
   attr[0].val.clusterDim.y = 1;
   attr[0].val.clusterDim.z = 1;
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
-  cfg.numAttrs = 1;
+  cfg.numAttrs = 2;
   return cudaLaunchKernelEx(&cfg, score_batch_split_kernel<LT, VEC>, p);
 }
 

@@ -88,6 +88,9 @@ __global__ void __launch_bounds__(kSelectThreads) buffer_record_kernel(
 }
 
 __global__ void state_init_kernel(stride_scan_state* s, int32_t n) {
+  // a programmatic dependent (the small-window and decode kernels) may be
+  // scheduled now; each of those waits for this grid before its first read
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
   const int32_t i = blockIdx.x * blockDim.x + threadIdx.x;
   if (i >= n) return;
   stride_scan_state z;

@@ -114,11 +114,11 @@ __global__ void combine_kernel(const float* __restrict__ parts, int32_t n_shards
 }
 
 // The scan on given log-probs, one tile of kScanTileRows consecutive rows per
-// CTA (one row per thread), tiles taken in ticket order.  Without a logit
-// pass to hide it, a lookback per row is what the time goes to (each row
-// waits on its predecessors' prefixes), so the rows of a tile are scanned
-// together in the CTA and only the tile takes part in the decoupled
-// lookback:
+// CTA (one row per thread), tiles taken in ticket order (by block index in a
+// small dependent grid, below).  Without a logit pass to hide it, a lookback
+// per row is what the time goes to (each row waits on its predecessors'
+// prefixes), so the rows of a tile are scanned together in the CTA and only
+// the tile takes part in the decoupled lookback:
 //   1. warps 0 and 1 find the tile's first turn and trajectory; the CTA
 //      stages the offsets of the next kScanTileRows + 1 turns and
 //      trajectories in shared memory and every thread finds its row's turn
@@ -244,7 +244,8 @@ __device__ __forceinline__ int smem_upper_le(const int64_t* a, int n, int64_t r)
 __global__ void __launch_bounds__(kScanTileRows) scan_logprobs_tile_kernel(const BatchParams p,
                                                                           const float* __restrict__ logp_s,
                                                                           const float* __restrict__ logp_t,
-                                                                          int64_t n_tiles, bool validate) {
+                                                                          int64_t n_tiles, bool validate,
+                                                                          bool by_ticket) {
   __shared__ int64_t s_turn_off[kScanTileRows + 1];
   __shared__ int64_t s_traj_row[kScanTileRows + 1];   // traj_row_off
   __shared__ int64_t s_traj_turn[kScanTileRows + 1];  // traj_turn_off, widened
@@ -259,11 +260,21 @@ __global__ void __launch_bounds__(kScanTileRows) scan_logprobs_tile_kernel(const
   __shared__ double s_prof[3 * STRIDE_PROFILE_BINS];
   __shared__ int64_t s_tile;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  // launched as a programmatic dependent of the kernel that wrote the
-  // log-probs: wait for it (a no-op otherwise)
-  asm volatile("griddepcontrol.wait;" ::: "memory");
-  if (tid == 0) s_tile = (int64_t)atomicAdd(p.ticket, 1u);
+  // Launched as a programmatic dependent of the kernel that wrote the
+  // log-probs (griddepcontrol.wait is a no-op otherwise).  That kernel
+  // waited for its own predecessors before letting this grid be scheduled,
+  // so the layout and the carried state may be read before the wait; the
+  // log-probs, the tile flags and the ticket only after it.  Tiles are
+  // taken in ticket order (a tile's lookback waits only on tiles taken
+  // before it, which are running or done) unless the grid is small enough
+  // to be resident at once, when the block index is the tile.
   if (tid < 3 * STRIDE_PROFILE_BINS) s_prof[tid] = 0.0;
+  if (by_ticket) {
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+    if (tid == 0) s_tile = (int64_t)atomicAdd(p.ticket, 1u);
+  } else if (tid == 0) {
+    s_tile = (int64_t)blockIdx.x;
+  }
   __syncthreads();
   const int64_t tile = s_tile;
   if (tile >= n_tiles) return;
@@ -273,11 +284,12 @@ __global__ void __launch_bounds__(kScanTileRows) scan_logprobs_tile_kernel(const
   const int64_t w = t0 + tid;  // this thread's window row
   const int64_t r = p.row_begin + w;
   const bool live = tid < n_here;
-  // the row's log-probs, in flight while the layout is looked up
+  // the row's log-probs, in flight while the layout is looked up (after
+  // the layout, below, when this grid has not waited yet)
   float lps = 0.f, lpt = 0.f;
-  if (live) {
-    lps = __ldg(logp_s + w);
-    lpt = __ldg(logp_t + w);
+  if (live && by_ticket) {
+    lps = __ldcg(logp_s + w);
+    lpt = __ldcg(logp_t + w);
   }
 
   // 1. the tile's first turn (warp 0) and first trajectory (warp 1), then
@@ -341,9 +353,28 @@ __global__ void __launch_bounds__(kScanTileRows) scan_logprobs_tile_kernel(const
     meta.bad = !(meta.turn_start <= r && r < meta.turn_end) || !(tr_start <= r && r < tr_end) ||
                !(tu0 <= turn && turn < tu1);
   }
+  // a seeded row's carried state, and lambda, before the wait
+  const bool seeded = live && ((w == 0) || (r == meta.traj_start) || meta.bad);
+  const int fturn = (live && r == meta.turn_start) ? 1 : 0;
+  double cum0 = 0.0, st0 = 0.0, sd0 = 0.0, sl0 = 0.0;
+  if (seeded && !meta.bad) {
+    const stride_scan_state* sp = p.state + meta.traj;
+    cum0 = __ldcg(&sp->cum);
+    st0 = fturn ? 0.0 : __ldcg(&sp->turn_sum_t);
+    sd0 = fturn ? 0.0 : __ldcg(&sp->turn_sum_d);
+    sl0 = fturn ? 0.0 : __ldcg(&sp->turn_sum_l);
+  }
+  const float lam = (live && !meta.bad) ? (p.lambda ? __ldg(p.lambda + meta.traj) : p.lambda_all) : 0.f;
+  if (!by_ticket) {
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+    if (live) {
+      lps = __ldcg(logp_s + w);
+      lpt = __ldcg(logp_t + w);
+    }
+  }
+
   TileElem x = {0.0, 0.0, 0.0, 0.0, 0};
   double c_before = 0.0, st_before = 0.0, e_sl = 0.0, ri_c = 0.0;
-  int fturn = 0;
   if (live) {
     const float nan = __int_as_float(0x7fc00000);
     if (meta.bad) {
@@ -359,20 +390,13 @@ __global__ void __launch_bounds__(kScanTileRows) scan_logprobs_tile_kernel(const
     const double ec = (p.mode == STRIDE_STOP_TURN_MEAN) ? (double)lpt / (double)(n_k > 0 ? n_k : 1) : (double)lpt;
     const double est = (double)lpt, esd = (double)dd, esl = (double)lps * (double)dd;
     e_sl = esl;
-    fturn = (r == meta.turn_start) ? 1 : 0;
     if (p.profile && !meta.bad) {
       const int jb = (int)((10 * (r - meta.turn_start)) / n_k);  // Observation 1 decile
       atomicAdd(s_prof + 3 * jb + 0, esd);
       atomicAdd(s_prof + 3 * jb + 1, est);
       atomicAdd(s_prof + 3 * jb + 2, 1.0);
     }
-    const bool seeded = (w == 0) || (r == meta.traj_start) || meta.bad;
     if (seeded && !meta.bad) {
-      const stride_scan_state* sp = p.state + meta.traj;
-      const double cum0 = __ldcg(&sp->cum);
-      const double st0 = fturn ? 0.0 : __ldcg(&sp->turn_sum_t);
-      const double sd0 = fturn ? 0.0 : __ldcg(&sp->turn_sum_d);
-      const double sl0 = fturn ? 0.0 : __ldcg(&sp->turn_sum_l);
       x = TileElem{cum0 + ec, st0 + est, sd0 + esd, sl0 + esl, kRestartSum | kRestartTurn};
       c_before = cum0;
       st_before = st0;
@@ -450,7 +474,6 @@ __global__ void __launch_bounds__(kScanTileRows) scan_logprobs_tile_kernel(const
     const int64_t n_k = meta.turn_end - meta.turn_start;
     const bool turn_last = (r == meta.turn_end - 1);
     const bool test = (p.mode == STRIDE_STOP_TOKEN_SUM) || turn_last;
-    const float lam = p.lambda ? __ldg(p.lambda + meta.traj) : p.lambda_all;
     cross = test && ri_c < (double)lam;
     const double before = (p.mode == STRIDE_STOP_TOKEN_SUM) ? c_before : c_before - st_before / (double)n_k;
     const bool kept = before >= (double)lam;
@@ -538,7 +561,16 @@ cudaError_t launch_scan_logprobs(const BatchParams& p, const float* logp_s, cons
   cfg.numAttrs = dependent ? 1 : 0;
   // the small-window kernel checks the layout itself (dependent launches)
   const bool validate = !dependent;
-  const cudaError_t e = cudaLaunchKernelEx(&cfg, scan_logprobs_tile_kernel, p, logp_s, logp_t, n_tiles, validate);
+  // A dependent grid of at most one CTA per SM is resident at once (the
+  // kernel it waits on always completes), so its tiles may go by block
+  // index: no ticket, and the layout is read before the wait.
+  int dev = 0;
+  cudaError_t qe = cudaSuccess;
+  const int sms = current_device_sms(&dev, &qe);
+  if (sms <= 0) return qe != cudaSuccess ? qe : cudaErrorInvalidDevice;
+  const bool by_ticket = !dependent || n_tiles > sms;
+  const cudaError_t e =
+      cudaLaunchKernelEx(&cfg, scan_logprobs_tile_kernel, p, logp_s, logp_t, n_tiles, validate, by_ticket);
   if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }
