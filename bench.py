@@ -61,7 +61,7 @@ def kernel_traffic_record() -> tuple[float | None, str]:
     summary, valid only while the kernel source is unchanged."""
     src = ROOT / "paper_2609_14636_gb300" / "csrc"
     h = hashlib.sha256()
-    for f in ("score_batch_stream.cu", "row_scan.cuh", "stride_device.cuh"):
+    for f in ("score_batch_stream.cu", "row_scan.cuh", "stride_device.cuh", "mbarrier.cuh"):
         h.update((src / f).read_bytes())
     digest = h.hexdigest()[:16]
     rec = ROOT / "profiles" / "score_batch_traffic.txt"

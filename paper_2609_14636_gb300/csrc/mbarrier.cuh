@@ -49,6 +49,16 @@ __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, uint64
   }
 }
 
+// mbar_wait for a whole warp (every lane calls it, converged): every lane
+// gets the same answer, false if any lane's wait ran out, so that the warp
+// leaves (or goes on) together and never reaches a warp-wide shuffle with
+// some of its lanes gone.
+__device__ __forceinline__ bool mbar_wait_warp(uint64_t* bar, uint32_t parity, uint64_t timeout_ns,
+                                               volatile int32_t* abort) {
+  const bool ok = mbar_wait(bar, parity, timeout_ns, abort);
+  return __all_sync(0xffffffffu, ok);
+}
+
 __device__ __forceinline__ void bulk_g2s(void* dst, const void* src, uint32_t bytes, uint64_t* bar,
                                          uint64_t policy) {
   asm volatile(

@@ -220,7 +220,7 @@ __global__ void __launch_bounds__(kStreamThreads, 1) score_batch_stream_kernel(c
     while (true) {
       const int s = (int)(it % kStages);
       const uint32_t k = it / kStages;
-      if (!mbar_wait(&sh.full[s], k & 1u, tmo, abort)) {
+      if (!mbar_wait_warp(&sh.full[s], k & 1u, tmo, abort)) {
         raise_abort(sh, p);
         break;
       }
@@ -260,7 +260,7 @@ __global__ void __launch_bounds__(kStreamThreads, 1) score_batch_stream_kernel(c
           mbar_arrive(&sh.red_done[q]);
         }
         if (cw == 0) {
-          if (!mbar_wait(&sh.red_done[q], use & 1u, tmo, abort)) {
+          if (!mbar_wait_warp(&sh.red_done[q], use & 1u, tmo, abort)) {
             raise_abort(sh, p);
             break;
           }
@@ -294,7 +294,7 @@ __global__ void __launch_bounds__(kStreamThreads, 1) score_batch_stream_kernel(c
     while (true) {
       const int q = (int)(seq % kSlots);
       const uint32_t use = (uint32_t)(seq / kSlots);
-      if (!mbar_wait(&sh.start[q], use & 1u, tmo, abort)) {
+      if (!mbar_wait_warp(&sh.start[q], use & 1u, tmo, abort)) {
         if (lane == 0) raise_abort(sh, p);
         break;
       }
@@ -328,7 +328,7 @@ __global__ void __launch_bounds__(kStreamThreads, 1) score_batch_stream_kernel(c
         lse_one(to_f32(trow[j]), tmT, tsT);
       }
       warp_merge2(tmS, tsS, tmT, tsT);
-      if (!mbar_wait(&sh.lse_ready[q], use & 1u, tmo, abort)) {
+      if (!mbar_wait_warp(&sh.lse_ready[q], use & 1u, tmo, abort)) {
         if (lane == 0) raise_abort(sh, p);
         break;
       }
@@ -369,6 +369,8 @@ __global__ void __launch_bounds__(kStreamThreads, 1) score_batch_stream_kernel(c
         }
       }
     }
+    // the warp leaves together (lanes whose waits ended differently agree)
+    ready = __all_sync(0xffffffffu, ready);
     if (!ready) break;
     const int64_t tile = sh.slot_tile[q];
     if (tile < 0) break;

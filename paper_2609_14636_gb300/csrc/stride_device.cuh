@@ -237,17 +237,27 @@ __device__ __forceinline__ void stream_pair(const LT* __restrict__ srow, const L
   }
 }
 
-// Warp-wide merge of two running pairs; every lane ends with the warp total.
+// Warp-wide merge of two running pairs; every lane ends with the warp total
+// (bit for bit the same in every lane: each butterfly step adds or takes the
+// larger of the same two values).  The warp's largest m first, then each
+// lane rescales its s to it once and the rescaled sums are added: two
+// exponentials per lane instead of one per pair and step.
 __device__ __forceinline__ void warp_merge2(float& mS, float& sS, float& mT, float& sT) {
+  float MS = mS, MT = mT;
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) {
-    float m2 = __shfl_xor_sync(0xffffffffu, mS, o);
-    float s2 = __shfl_xor_sync(0xffffffffu, sS, o);
-    lse_merge(mS, sS, m2, s2);
-    m2 = __shfl_xor_sync(0xffffffffu, mT, o);
-    s2 = __shfl_xor_sync(0xffffffffu, sT, o);
-    lse_merge(mT, sT, m2, s2);
+    MS = fmaxf(MS, __shfl_xor_sync(0xffffffffu, MS, o));
+    MT = fmaxf(MT, __shfl_xor_sync(0xffffffffu, MT, o));
   }
+  sS *= ex2((mS - MS) * kLog2e);
+  sT *= ex2((mT - MT) * kLog2e);
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    sS += __shfl_xor_sync(0xffffffffu, sS, o);
+    sT += __shfl_xor_sync(0xffffffffu, sT, o);
+  }
+  mS = MS;
+  mT = MT;
 }
 
 __device__ __forceinline__ uint64_t globaltimer_ns() {

@@ -68,13 +68,18 @@ def _scan(stride, ls, lt, lay, mode, lam, windows=None):
                 status=int(status.item()), profile=prof.cpu().numpy())
 
 
-@pytest.mark.parametrize("bounds_kind", ["4_equal", "3_ragged"])
+@pytest.mark.parametrize("bounds_kind", ["4_equal", "3_ragged", "aligned_with_tail"])
 def test_shards_combine_to_full_rows(stride, bounds_kind):
+    """4_equal: 16-byte-aligned shards of whole vectors; 3_ragged: shards
+    starting off the 16-byte grid; aligned_with_tail: an aligned shard whose
+    width leaves 3 logits past its last whole vector, then an unaligned
+    one."""
     import torch
 
     V = 151_936
     lay, S, T, tok = _case(61, V)
-    bounds = [0, 37_984, 75_968, 113_952, V] if bounds_kind == "4_equal" else [0, 50_001, 100_003, V]
+    bounds = {"4_equal": [0, 37_984, 75_968, 113_952, V], "3_ragged": [0, 50_001, 100_003, V],
+              "aligned_with_tail": [0, 40_000, 80_003, V]}[bounds_kind]
     St, Tt = to_dev(S), to_dev(T)
     tk = torch.from_numpy(tok).cuda()
     ls, lt, status = _sharded_logprobs(stride, St, Tt, tk, bounds)
