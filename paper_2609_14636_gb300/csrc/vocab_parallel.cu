@@ -20,8 +20,25 @@
 
 namespace stride {
 
-constexpr int kPartialThreads = 256;
+// Shard-pass launch shape (build defines, for sweeps): threads per CTA,
+// 16-byte loads in flight per thread and tensor, and CTAs per SM promised
+// to the register allocator.  A sweep on GB300 (4 shards of the batch-
+// scoring rows, 37,984 bf16 logits per shard row; ms for the 4 passes):
+// 128 threads x 4 loads at 8 CTAs per SM (58 registers) 12.25; 256 x 3 at
+// 8 per SM 12.26; 128 x 4 unbounded (7 per SM) 12.30; 256 x 4 at 4 per SM
+// 12.48; 256 x 2 12.82; 256 x 4 unbounded (66 registers, 3 per SM) 13.03.
+#ifndef STRIDE_PARTIAL_THREADS
+#define STRIDE_PARTIAL_THREADS 128
+#endif
+#ifndef STRIDE_PARTIAL_UNROLL
+#define STRIDE_PARTIAL_UNROLL 4
+#endif
+#ifndef STRIDE_PARTIAL_MIN_BLOCKS
+#define STRIDE_PARTIAL_MIN_BLOCKS 8
+#endif
+constexpr int kPartialThreads = STRIDE_PARTIAL_THREADS;
 constexpr int kPartialWarps = kPartialThreads / 32;
+static_assert(kPartialThreads % 32 == 0 && kPartialWarps <= 32, "whole warps, at most 32");
 
 struct PartialParams {
   const void* S;
@@ -39,14 +56,14 @@ struct PartialParams {
 // One CTA per row: (m, s) of S and T over this shard's columns, and the
 // gathered logits when the token is one of them (NaN otherwise).
 template <typename LT, bool VEC>
-__global__ void __launch_bounds__(kPartialThreads) partial_lse_kernel(const PartialParams p) {
+__global__ void __launch_bounds__(kPartialThreads, STRIDE_PARTIAL_MIN_BLOCKS) partial_lse_kernel(const PartialParams p) {
   __shared__ float s_red[4][kPartialWarps];
   const int64_t r = blockIdx.x;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const LT* srow = reinterpret_cast<const LT*>(p.S) + r * p.ld;
   const LT* trow = reinterpret_cast<const LT*>(p.T) + r * p.ld;
   float mS = kMaxStart, sS = 0.f, mT = kMaxStart, sT = 0.f;
-  stream_pair<LT, VEC, 4>(srow, trow, 0, p.V_shard, tid, kPartialThreads, mS, sS, mT, sT);
+  stream_pair<LT, VEC, STRIDE_PARTIAL_UNROLL>(srow, trow, 0, p.V_shard, tid, kPartialThreads, mS, sS, mT, sT);
   warp_merge2(mS, sS, mT, sT);
   if (lane == 0) {
     s_red[0][warp] = mS;
