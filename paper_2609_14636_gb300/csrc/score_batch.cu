@@ -369,7 +369,11 @@ cudaError_t launch_score_batch(const BatchParams& p, int dtype, bool vec, size_t
     if (e != cudaSuccess) return e;
   }
   const int per_vec = dtype == STRIDE_DTYPE_BF16 ? 8 : 4;
-  if (vec && p.V >= per_vec && !f_rows) return launch_score_batch_stream(p, dtype, stream);
+  // (the persistent kernel counts a row's bytes in 32 bits: rows of up to
+  // 2 GB, far beyond any vocabulary, take it)
+  const int64_t row_bytes = (int64_t)p.V * (dtype == STRIDE_DTYPE_BF16 ? 2 : 4);
+  if (vec && p.V >= per_vec && row_bytes <= ((int64_t)1 << 31) && !f_rows)
+    return launch_score_batch_stream(p, dtype, stream);
   const dim3 grid((unsigned)p.n_rows), block(kBatchThreads);
   if (dtype == STRIDE_DTYPE_BF16) {
     if (vec)
