@@ -7,7 +7,10 @@ configurations the library is used in, against the oracle on every row.
   with the carried state, then the restart choice over its turn statistics
   with Bernoulli(0.5) and Bernoulli(0.9) masks, alpha = -inf and -6.0;
 * multi-teacher (128 x 12 turns, 436,156 rows, two teacher streams): streamed
-  in 16,384-row windows.
+  in 16,384-row windows;
+* the batch-scoring rows again through the vocabulary-sharded path (the
+  bench's 4 shards: partial passes, combine, scan on log-probs), on the same
+  resident logits.
 
 The oracle scores every row (fp64, all host cores) from device->host copies
 of the same logits."""
@@ -62,9 +65,39 @@ def oracle_rows(copier, S, T, tok, out_rows: dict, r0: int):
             out_rows[k][r0 + a:r0 + b] = o[k]
 
 
-def stream_and_score(stride, w, lam, chunk_rows, resident=False):
+def sharded_scan(stride, S, T, tok, offs, lay, lam, n_shards):
+    """The vocabulary-sharded path on resident logits: stride_partial_lse on
+    n_shards column ranges (16-byte-aligned cuts, as the bench takes them),
+    stride_combine_partials, stride_scan_logprobs over the whole window."""
+    import torch
+
+    R, V = S.shape
+    cuts = [((k * V // n_shards) // 8) * 8 for k in range(n_shards)] + [V]
+    dev = S.device
+    parts = torch.empty((n_shards, R, 6), dtype=torch.float32, device=dev)
+    status = torch.zeros(1, dtype=torch.int32, device=dev)
+    for k in range(n_shards):
+        c0, c1 = cuts[k], cuts[k + 1]
+        stride.stride_partial_lse(S[:, c0:c1], T[:, c0:c1], tok, c0, parts[k], status, V_shard=c1 - c0)
+    out = {k: torch.empty(R, dtype=torch.float32, device=dev) for k in ("logp_s", "logp_t", "lse_s", "lse_t", "opd")}
+    stride.stride_combine_partials(parts, out["logp_s"], out["logp_t"], out["lse_s"], out["lse_t"], dev_status=status)
+    st = stride.new_state(lay.n_traj)
+    ts = stride.new_turn_stats(lay.n_turns)
+    ws = torch.empty(stride.stride_score_batch_workspace_size(R), dtype=torch.uint8, device=dev)
+    stride.stride_scan_logprobs(out["logp_s"], out["logp_t"], *offs, 0, R, stride.TURN_MEAN, float(lam), st,
+                                opd=out["opd"], turn_stats=ts, dev_status=status, workspace=ws)
+    torch.cuda.synchronize()
+    g = {k: v.cpu().numpy() for k, v in out.items()}
+    g["state"] = stride.state_to_numpy(st)[: lay.n_traj]
+    g["turn_stats"] = stride.turn_stats_to_numpy(ts)[: lay.n_turns]
+    g["status"] = int(status.item())
+    return g
+
+
+def stream_and_score(stride, w, lam, chunk_rows, resident=False, vocab_shards=0):
     """Generate the workload window by window on the GPU, score each window
-    with the carried state, and run the oracle on the same rows."""
+    with the carried state, and run the oracle on the same rows (and, on a
+    resident workload, the vocabulary-sharded path too)."""
     import torch
 
     lay = w.layout
@@ -103,6 +136,8 @@ def stream_and_score(stride, w, lam, chunk_rows, resident=False):
     g["turn_stats"] = stride.turn_stats_to_numpy(ts)[: lay.n_turns]
     g["status"] = int(status.item())
     g["profile"] = prof.cpu().numpy()
+    if resident and vocab_shards:
+        g["sharded"] = sharded_scan(stride, S, T, tok, offs, lay, lam, vocab_shards)
     sc = oracle.scan_batch(o["logp_t"], o["d"], lay.traj_row_off, lay.turn_row_off, lay.traj_turn_off,
                            oracle.TURN_MEAN, float(np.float32(lam)), logp_s=o["logp_s"])
     o.update(sc)
@@ -120,8 +155,10 @@ def _check(g, o, lay, lam, expect_frac):
 def test_full_batch_scoring_resident(stride):
     w = synth.batch_scoring()
     cal = synth.load_calibration(w.name)
-    g, o = stream_and_score(stride, w, cal["lambda"], None, resident=True)
+    g, o = stream_and_score(stride, w, cal["lambda"], None, resident=True, vocab_shards=4)
     _check(g, o, w.layout, cal["lambda"], cal["early_stop_fraction"])
+    # the same rows through the vocabulary-sharded path
+    _check(g["sharded"], o, w.layout, cal["lambda"], cal["early_stop_fraction"])
 
 
 def test_full_long_agentic_chunked_then_select(stride):
