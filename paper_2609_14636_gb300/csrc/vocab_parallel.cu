@@ -13,7 +13,6 @@
 // the fused kernels' decoupled lookback (row_scan.cuh) between tiles.
 #include <math.h>
 
-#include "dfloat.cuh"
 #include "row_scan.cuh"
 #include "stride.h"
 #include "stride_device.cuh"
@@ -163,46 +162,36 @@ constexpr int kScanTileWarps = kScanTileRows / 32;
 constexpr int kRestartTurn = 1;  // st, sd, sl restart at this row
 constexpr int kRestartSum = 2;   // c restarts (a seeded row)
 
-// The tile's sums are double-floats (dfloat.cuh): the published aggregates
-// and prefixes, the carried state and the outputs stay fp64.
 struct TileElem {
-  dfloat c, st, sd, sl;
+  double c, st, sd, sl;
   int flags;
 };
 
 __device__ __forceinline__ TileElem tile_combine(const TileElem& a, const TileElem& b) {
   TileElem r;
-  r.c = (b.flags & kRestartSum) ? b.c : df_add(a.c, b.c);
-  r.st = (b.flags & kRestartTurn) ? b.st : df_add(a.st, b.st);
-  r.sd = (b.flags & kRestartTurn) ? b.sd : df_add(a.sd, b.sd);
-  r.sl = (b.flags & kRestartTurn) ? b.sl : df_add(a.sl, b.sl);
+  r.c = (b.flags & kRestartSum) ? b.c : a.c + b.c;
+  r.st = (b.flags & kRestartTurn) ? b.st : a.st + b.st;
+  r.sd = (b.flags & kRestartTurn) ? b.sd : a.sd + b.sd;
+  r.sl = (b.flags & kRestartTurn) ? b.sl : a.sl + b.sl;
   r.flags = a.flags | b.flags;
   return r;
 }
 
 __device__ __forceinline__ TileElem tile_shfl_up(const TileElem& v, int d) {
   TileElem o;
-  o.c = df_shfl_up(v.c, d);
-  o.st = df_shfl_up(v.st, d);
-  o.sd = df_shfl_up(v.sd, d);
-  o.sl = df_shfl_up(v.sl, d);
+  o.c = __shfl_up_sync(0xffffffffu, v.c, d);
+  o.st = __shfl_up_sync(0xffffffffu, v.st, d);
+  o.sd = __shfl_up_sync(0xffffffffu, v.sd, d);
+  o.sl = __shfl_up_sync(0xffffffffu, v.sl, d);
   o.flags = __shfl_up_sync(0xffffffffu, v.flags, d);
   return o;
-}
-
-__device__ __forceinline__ TileElem tile_from_scan(const ScanElem& e) {
-  return TileElem{df_from_double(e.c), df_from_double(e.st), df_from_double(e.sd), df_from_double(e.sl), 0};
-}
-
-__device__ __forceinline__ ScanElem scan_from_tile(const TileElem& e, int fturn) {
-  return ScanElem{df_to_double(e.c), df_to_double(e.st), df_to_double(e.sd), df_to_double(e.sl), fturn};
 }
 
 // Per-trajectory sums of the tile's rows for the trajectory's record: the
 // retained rows' loss terms and count, and whether a row crossed lambda.
 // Restarts at a trajectory's first row.
 struct TrajElem {
-  dfloat loss;
+  double loss;
   int count;
   int crossed;
   int restart;
@@ -210,12 +199,12 @@ struct TrajElem {
 
 __device__ __forceinline__ TrajElem traj_combine(const TrajElem& a, const TrajElem& b) {
   if (b.restart) return b;
-  return TrajElem{df_add(a.loss, b.loss), a.count + b.count, a.crossed | b.crossed, a.restart};
+  return TrajElem{a.loss + b.loss, a.count + b.count, a.crossed | b.crossed, a.restart};
 }
 
 __device__ __forceinline__ TrajElem traj_shfl_up(const TrajElem& v, int d) {
   TrajElem o;
-  o.loss = df_shfl_up(v.loss, d);
+  o.loss = __shfl_up_sync(0xffffffffu, v.loss, d);
   o.count = __shfl_up_sync(0xffffffffu, v.count, d);
   o.crossed = __shfl_up_sync(0xffffffffu, v.crossed, d);
   o.restart = __shfl_up_sync(0xffffffffu, v.restart, d);
@@ -401,9 +390,8 @@ __global__ void __launch_bounds__(kScanTileRows) scan_logprobs_tile_kernel(const
     }
   }
 
-  const dfloat dz = df_from(0.f);
-  TileElem x = {dz, dz, dz, dz, 0};
-  dfloat c_before = dz, st_before = dz, e_sl = dz, ri_c = dz;
+  TileElem x = {0.0, 0.0, 0.0, 0.0, 0};
+  double c_before = 0.0, st_before = 0.0, e_sl = 0.0, ri_c = 0.0;
   if (live) {
     const float nan = __int_as_float(0x7fc00000);
     if (meta.bad) {
@@ -416,24 +404,19 @@ __global__ void __launch_bounds__(kScanTileRows) scan_logprobs_tile_kernel(const
     const float dd = lps - lpt;
     if (p.out.opd) p.out.opd[w] = dd;
     const int64_t n_k = meta.turn_end - meta.turn_start;
-    // the row's terms: log pi_T (over n_k in turn mode), d, and logp_S * d
-    // (an exact product)
-    const dfloat ec = (p.mode == STRIDE_STOP_TURN_MEAN) ? df_div_count(df_from(lpt), (float)(n_k > 0 ? n_k : 1))
-                                                        : df_from(lpt);
-    const dfloat est = df_from(lpt), esd = df_from(dd), esl = df_mul_ff(lps, dd);
+    const double ec = (p.mode == STRIDE_STOP_TURN_MEAN) ? (double)lpt / (double)(n_k > 0 ? n_k : 1) : (double)lpt;
+    const double est = (double)lpt, esd = (double)dd, esl = (double)lps * (double)dd;
     e_sl = esl;
     if (p.profile && !meta.bad) {
       const int jb = (int)((10 * (r - meta.turn_start)) / n_k);  // Observation 1 decile
-      atomicAdd(s_prof + 3 * jb + 0, (double)dd);
-      atomicAdd(s_prof + 3 * jb + 1, (double)lpt);
+      atomicAdd(s_prof + 3 * jb + 0, esd);
+      atomicAdd(s_prof + 3 * jb + 1, est);
       atomicAdd(s_prof + 3 * jb + 2, 1.0);
     }
     if (seeded && !meta.bad) {
-      const dfloat c0d = df_from_double(cum0);
-      x = TileElem{df_add(c0d, ec), df_add(df_from_double(st0), est), df_add(df_from_double(sd0), esd),
-                   df_add(df_from_double(sl0), esl), kRestartSum | kRestartTurn};
-      c_before = c0d;
-      st_before = df_from_double(st0);
+      x = TileElem{cum0 + ec, st0 + est, sd0 + esd, sl0 + esl, kRestartSum | kRestartTurn};
+      c_before = cum0;
+      st_before = st0;
     } else if (seeded) {
       x = TileElem{ec, est, esd, esl, kRestartSum | kRestartTurn};  // NaN: nothing after a bad row is meaningful
     } else {
@@ -443,13 +426,13 @@ __global__ void __launch_bounds__(kScanTileRows) scan_logprobs_tile_kernel(const
   }
 
   // 3. segmented inclusive scan over the tile
-  const TileElem tile_id = {dz, dz, dz, dz, 0};
+  const TileElem tile_id = {0.0, 0.0, 0.0, 0.0, 0};
   TileElem tile_incl, tile_excl;
   block_scan(x, tile_id, lane, warp, s_wtot, s_wpre, tile_incl, tile_excl);
 
   // 4. publish the tile's aggregate, fold predecessors, publish its prefix
   if (tid == (int)(n_here - 1)) {
-    const ScanElem agg = scan_from_tile(tile_incl, tile_incl.flags & kRestartTurn);
+    ScanElem agg{tile_incl.c, tile_incl.st, tile_incl.sd, tile_incl.sl, tile_incl.flags & kRestartTurn};
     if (tile_incl.flags & kRestartSum) {
       publish(p.incl + tile, p.flags + tile * kFlagStride, agg, kStIncl);
     } else {
@@ -461,16 +444,17 @@ __global__ void __launch_bounds__(kScanTileRows) scan_logprobs_tile_kernel(const
   __syncthreads();
   if (warp == 0) {
     const TileElem agg = s_agg;
-    TileElem pre = {dz, dz, dz, dz, 0};
+    TileElem pre = {0.0, 0.0, 0.0, 0.0, 0};
     bool timed_out = false;
     // The rows before the tile's first seeded row need the predecessors' sum
     // (a tile whose first row is seeded needs nothing).
     if (!(__shfl_sync(0xffffffffu, x.flags, 0) & kRestartSum)) {
       const ScanElem e = lookback(p, tile, lane, timed_out);
-      pre = tile_from_scan(e);
+      pre = TileElem{e.c, e.st, e.sd, e.sl, 0};
       if (lane == 0 && !(agg.flags & kRestartSum)) {
         const TileElem inc = tile_combine(pre, agg);
-        publish(p.incl + tile, p.flags + tile * kFlagStride, scan_from_tile(inc, 1), kStIncl);
+        ScanElem ie{inc.c, inc.st, inc.sd, inc.sl, 1};
+        publish(p.incl + tile, p.flags + tile * kFlagStride, ie, kStIncl);
       }
     }
     if (lane == 0) {
@@ -487,17 +471,12 @@ __global__ void __launch_bounds__(kScanTileRows) scan_logprobs_tile_kernel(const
     if (!(x.flags & 4)) {
       const TileElem re = tile_combine(pre, tile_excl);
       c_before = re.c;
-      st_before = fturn ? dz : re.st;
+      st_before = fturn ? 0.0 : re.st;
     }
-    // turn statistics and carried state, written by a turn's last row and a
-    // trajectory's (or the window's) last row (row_tail does nothing else
-    // here: the stop records and losses follow below)
-    const bool timed_out = (s_flags & 1) != 0;
-    if (timed_out || r == meta.turn_end - 1 || r == meta.traj_end - 1 || r == p.row_end - 1) {
-      RowCarry rc;
-      rc.e = ScanElem{0.0, 0.0, 0.0, df_to_double(e_sl), fturn};
-      row_tail(p, r, meta, rc, scan_from_tile(ri, 1), 0.0, 0.0, timed_out, true);
-    }
+    RowCarry rc;
+    rc.e = ScanElem{0.0, 0.0, 0.0, e_sl, fturn};
+    const ScanElem si{ri.c, ri.st, ri.sd, ri.sl, 1};
+    row_tail(p, r, meta, rc, si, c_before, st_before, (s_flags & 1) != 0, true);
     ri_c = ri.c;
   }
 
@@ -506,20 +485,18 @@ __global__ void __launch_bounds__(kScanTileRows) scan_logprobs_tile_kernel(const
   //    the stop (the running sum never rises, so it is the trajectory's
   //    first crossing unless an earlier tile's is lower), and the last row
   //    of a trajectory here adds its retained rows' loss and count.
-  TrajElem te = {df_from(0.f), 0, 0, 1};
+  TrajElem te = {0.0, 0, 0, 1};
   bool cross = false;
   if (live && !meta.bad) {
     const int64_t n_k = meta.turn_end - meta.turn_start;
     const bool turn_last = (r == meta.turn_end - 1);
     const bool test = (p.mode == STRIDE_STOP_TOKEN_SUM) || turn_last;
-    cross = test && df_lt(ri_c, lam);
-    const dfloat before = (p.mode == STRIDE_STOP_TOKEN_SUM)
-                              ? c_before
-                              : df_add(c_before, df_neg(df_div_count(st_before, (float)n_k)));
-    const bool kept = df_ge(before, lam);
-    te = TrajElem{kept ? e_sl : dz, kept ? 1 : 0, cross ? 1 : 0, r == meta.traj_start ? 1 : 0};
+    cross = test && ri_c < (double)lam;
+    const double before = (p.mode == STRIDE_STOP_TOKEN_SUM) ? c_before : c_before - st_before / (double)n_k;
+    const bool kept = before >= (double)lam;
+    te = TrajElem{kept ? e_sl : 0.0, kept ? 1 : 0, cross ? 1 : 0, r == meta.traj_start ? 1 : 0};
   }
-  const TrajElem traj_id = {dz, 0, 0, 0};
+  const TrajElem traj_id = {0.0, 0, 0, 0};
   TrajElem t_incl, t_excl;
   block_scan(te, traj_id, lane, warp, s_ttot, s_tpre, t_incl, t_excl);
   if (live && !meta.bad) {
@@ -530,7 +507,7 @@ __global__ void __launch_bounds__(kScanTileRows) scan_logprobs_tile_kernel(const
       sp->stopped = 1;
     }
     if ((r == meta.traj_end - 1 || tid == (int)(n_here - 1)) && t_incl.count > 0) {
-      atomicAdd(&sp->loss, df_to_double(t_incl.loss));
+      atomicAdd(&sp->loss, t_incl.loss);
       atomicAdd(reinterpret_cast<unsigned long long*>(&sp->loss_tokens), (unsigned long long)t_incl.count);
     }
   }

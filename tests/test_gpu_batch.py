@@ -212,6 +212,28 @@ def test_masked_vocab_entries(stride, kernel):
     assert g["logp_s"][3] == -np.inf
 
 
+@pytest.mark.parametrize("mode", [0, 1])
+def test_masked_teacher_token_stops_at_minus_inf(stride, kernel, mode):
+    """A sampled token whose teacher logit is -inf: log pi_T = -inf, so the
+    running sum is -inf from that row (token mode) or that turn's end (turn
+    mode) on, and the trajectory stops there, as in the fp64 oracle."""
+    lay = synth.layout_from_turn_lengths([[6, 6, 4], [5, 7]])
+    V = 5000
+    S, T, tok = _bf16_rows(43, lay.rows, V)
+    T[8, 2000:2500] = 0xFF80  # trajectory 0, turn 1, its third row
+    tok[8] = 2100
+    g = run_batch(stride, S, T, tok, lay, mode, -1e30)
+    o = oracle_batch(S, T, tok, lay, mode, -1e30)
+    assert g["logp_t"][8] == -np.inf and o["logp_t"][8] == -np.inf
+    st = g["state"]
+    assert int(st["stop_turn"][0]) == 1
+    assert int(st["stop_row"][0]) == (8 if mode == 1 else 11)
+    assert int(st["stop_row"][1]) == -1 and int(st["stop_turn"][1]) == -1
+    ts = g["turn_stats"]
+    assert ts["sum_t"][1] == -np.inf and o["turn_sum_t"][1] == -np.inf
+    assert ts["sum_t"][3] == pytest.approx(o["turn_sum_t"][3], rel=1e-5)
+
+
 def test_token_out_of_range_sets_status(stride, kernel):
     lay = synth.layout_from_turn_lengths([[4], [3]])
     S, T, tok = _bf16_rows(51, lay.rows, 1000)
