@@ -145,9 +145,9 @@ __global__ void __launch_bounds__(kSplitThreads, kSplitBlocksPerSm)
   asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
   if (blockIdx.x == 0) {
     // What the scan needs at zero: its tile ticket (the header's second
-    // word) and one flag per 256-row tile.  The scan reads them only after
-    // this grid has completed.
-    const int64_t n_tiles = (p.n_rows + 255) / 256;
+    // word) and one flag per tile of kScanTileRowsDependent rows.  The scan
+    // reads them only after this grid has completed.
+    const int64_t n_tiles = (p.n_rows + kScanTileRowsDependent - 1) / kScanTileRowsDependent;
     for (int64_t t = threadIdx.x; t < n_tiles; t += blockDim.x) p.flags[t * kFlagStride] = 0u;
     if (threadIdx.x == 0) p.ticket[1] = 0u;
   }

@@ -22,6 +22,26 @@ struct alignas(32) ScanSlot {
 // 1,024 rows scored 3-12 % faster with the flags spread out.
 constexpr int kFlagStride = 32;
 
+// Rows per tile (and threads per CTA) of the tiled scan on log-probs (build
+// defines, for sweeps): on its own (stride_scan_logprobs, the sharded path)
+// and as the programmatic dependent that completes a small window.  A sweep
+// on GB300 (one size for both): the 148,909-row scan took 52.8 / 51.2 / 49.2
+// / 49.6 us with tiles of 64 / 128 / 256 / 512 rows, the 512-row tiny step
+// 36.6 / 36.7 / 37.4 / 39.0 us: many small tiles finish a small window's
+// chain sooner, larger ones run a long scan with fewer lookbacks.
+#ifndef STRIDE_SCAN_TILE_ROWS
+#define STRIDE_SCAN_TILE_ROWS 256
+#endif
+#ifndef STRIDE_SCAN_TILE_ROWS_DEPENDENT
+#define STRIDE_SCAN_TILE_ROWS_DEPENDENT 128
+#endif
+constexpr int kScanTileRows = STRIDE_SCAN_TILE_ROWS;
+constexpr int kScanTileRowsDependent = STRIDE_SCAN_TILE_ROWS_DEPENDENT;
+static_assert(kScanTileRows % 32 == 0 && kScanTileRows >= 64 && kScanTileRows <= 1024,
+              "whole warps, 2 to 32 of them");
+static_assert(kScanTileRowsDependent % 32 == 0 && kScanTileRowsDependent >= 64 && kScanTileRowsDependent <= 1024,
+              "whole warps, 2 to 32 of them");
+
 struct BatchParams {
   const void* S;
   const void* T;

@@ -130,8 +130,9 @@ __global__ void combine_kernel(const float* __restrict__ parts, int32_t n_shards
   if (lse_t) lse_t[r] = lt;
 }
 
-// The scan on given log-probs, one tile of kScanTileRows consecutive rows per
-// CTA (one row per thread), tiles taken in ticket order (by block index in a
+// The scan on given log-probs, one tile of TILE consecutive rows per CTA (one
+// row per thread; kScanTileRows on its own, kScanTileRowsDependent after the
+// small-window kernel), tiles taken in ticket order (by block index in a
 // small dependent grid, below).  Without a logit pass to hide it, a lookback
 // per row is what the time goes to (each row waits on its predecessors'
 // prefixes), so the rows of a tile are scanned together in the CTA and only
@@ -157,8 +158,6 @@ __global__ void combine_kernel(const float* __restrict__ parts, int32_t n_shards
 //      trajectory's retained loss and first crossing in the tile, so the
 //      trajectory's record takes one update per tile instead of one per row
 //      (the rows of a token-sum segment below lambda all contended for it).
-constexpr int kScanTileRows = 256;
-constexpr int kScanTileWarps = kScanTileRows / 32;
 constexpr int kRestartTurn = 1;  // st, sd, sl restart at this row
 constexpr int kRestartSum = 2;   // c restarts (a seeded row)
 
@@ -217,10 +216,10 @@ __device__ __forceinline__ TileElem elem_shfl_up(const TileElem& v, int d) { ret
 __device__ __forceinline__ TrajElem elem_shfl_up(const TrajElem& v, int d) { return traj_shfl_up(v, d); }
 
 // Inclusive and exclusive scan of one element per thread over the CTA's
-// kScanTileRows threads, in thread order: warp shuffles, then warp 0 scans
-// the warps' totals once (each thread then combines with one prefix).
-// `id` is the identity; s_tot and s_pre hold kScanTileWarps elements.
-template <typename E>
+// WARPS warps, in thread order: warp shuffles, then warp 0 scans the warps'
+// totals once (each thread then combines with one prefix).  `id` is the
+// identity; s_tot and s_pre hold WARPS elements.
+template <int WARPS, typename E>
 __device__ __forceinline__ void block_scan(const E& v, const E& id, int lane, int warp, E* s_tot, E* s_pre,
                                            E& incl_out, E& excl_out) {
   E incl = v;
@@ -233,14 +232,14 @@ __device__ __forceinline__ void block_scan(const E& v, const E& id, int lane, in
   if (lane == 31) s_tot[warp] = incl;
   __syncthreads();
   if (warp == 0) {
-    E t = lane < kScanTileWarps ? s_tot[lane] : id;
+    E t = lane < WARPS ? s_tot[lane] : id;
 #pragma unroll
-    for (int d = 1; d < kScanTileWarps; d <<= 1) {
+    for (int d = 1; d < WARPS; d <<= 1) {
       const E o = elem_shfl_up(t, d);
       if (lane >= d) t = elem_combine(o, t);
     }
     const E e = elem_shfl_up(t, 1);
-    if (lane < kScanTileWarps) s_pre[lane] = (lane == 0) ? id : e;
+    if (lane < WARPS) s_pre[lane] = (lane == 0) ? id : e;
   }
   __syncthreads();
   const E wpre = s_pre[warp];
@@ -258,19 +257,21 @@ __device__ __forceinline__ int smem_upper_le(const int64_t* a, int n, int64_t r)
   return lo;
 }
 
-__global__ void __launch_bounds__(kScanTileRows) scan_logprobs_tile_kernel(const BatchParams p,
+template <int TILE>
+__global__ void __launch_bounds__(TILE) scan_logprobs_tile_kernel(const BatchParams p,
                                                                           const float* __restrict__ logp_s,
                                                                           const float* __restrict__ logp_t,
                                                                           int64_t n_tiles, bool validate,
                                                                           bool by_ticket) {
-  __shared__ int64_t s_turn_off[kScanTileRows + 1];
-  __shared__ int64_t s_traj_row[kScanTileRows + 1];   // traj_row_off
-  __shared__ int64_t s_traj_turn[kScanTileRows + 1];  // traj_turn_off, widened
+  constexpr int kWarps = TILE / 32;
+  __shared__ int64_t s_turn_off[TILE + 1];
+  __shared__ int64_t s_traj_row[TILE + 1];   // traj_row_off
+  __shared__ int64_t s_traj_turn[TILE + 1];  // traj_turn_off, widened
   __shared__ int64_t s_first[2];                      // first turn, first trajectory of the tile
-  __shared__ TileElem s_wtot[kScanTileWarps];
-  __shared__ TileElem s_wpre[kScanTileWarps];
-  __shared__ TrajElem s_ttot[kScanTileWarps];
-  __shared__ TrajElem s_tpre[kScanTileWarps];
+  __shared__ TileElem s_wtot[kWarps];
+  __shared__ TileElem s_wpre[kWarps];
+  __shared__ TrajElem s_ttot[kWarps];
+  __shared__ TrajElem s_tpre[kWarps];
   __shared__ TileElem s_excl;
   __shared__ TileElem s_agg;
   __shared__ int s_flags;  // bit 0: lookback timed out
@@ -295,8 +296,8 @@ __global__ void __launch_bounds__(kScanTileRows) scan_logprobs_tile_kernel(const
   __syncthreads();
   const int64_t tile = s_tile;
   if (tile >= n_tiles) return;
-  const int64_t t0 = tile * kScanTileRows;           // first window row of the tile
-  const int64_t n_here = min((int64_t)kScanTileRows, p.n_rows - t0);
+  const int64_t t0 = tile * TILE;           // first window row of the tile
+  const int64_t n_here = min((int64_t)TILE, p.n_rows - t0);
   const int64_t r0 = p.row_begin + t0;
   const int64_t w = t0 + tid;  // this thread's window row
   const int64_t r = p.row_begin + w;
@@ -310,7 +311,7 @@ __global__ void __launch_bounds__(kScanTileRows) scan_logprobs_tile_kernel(const
   }
 
   // 1. the tile's first turn (warp 0) and first trajectory (warp 1), then
-  //    the offsets of the next kScanTileRows + 1 of each in shared memory
+  //    the offsets of the next TILE + 1 of each in shared memory
   if (warp == 0) {
     const bool ok = p.n_turns > 0 && __ldg(p.turn_row_off) <= r0;
     const int64_t k0 = ok ? warp_upper_le(p.turn_row_off, 0, p.n_turns - 1, r0, lane) : 0;
@@ -323,7 +324,7 @@ __global__ void __launch_bounds__(kScanTileRows) scan_logprobs_tile_kernel(const
   __syncthreads();
   const int64_t k0 = s_first[0], i0 = s_first[1];
   if (k0 >= 0 && i0 >= 0) {
-    for (int j = tid; j <= kScanTileRows; j += kScanTileRows) {
+    for (int j = tid; j <= TILE; j += TILE) {
       s_turn_off[j] = __ldg(p.turn_row_off + min(k0 + j, (int64_t)p.n_turns));
       s_traj_row[j] = __ldg(p.traj_row_off + min(i0 + j, (int64_t)p.n_traj));
       s_traj_turn[j] = __ldg(p.traj_turn_off + min(i0 + j, (int64_t)p.n_traj));
@@ -339,14 +340,14 @@ __global__ void __launch_bounds__(kScanTileRows) scan_logprobs_tile_kernel(const
   meta.local_turn = 0;
   meta.traj_start = meta.traj_end = meta.turn_start = meta.turn_end = 0;
   if (live && k0 >= 0 && i0 >= 0) {
-    const int nk = (int)min((int64_t)kScanTileRows, (int64_t)p.n_turns - k0);
+    const int nk = (int)min((int64_t)TILE, (int64_t)p.n_turns - k0);
     const int j = smem_upper_le(s_turn_off, nk, r);
-    const int ni = (int)min((int64_t)kScanTileRows, (int64_t)p.n_traj - i0);
+    const int ni = (int)min((int64_t)TILE, (int64_t)p.n_traj - i0);
     int q = smem_upper_le(s_traj_row, ni, r);
     int64_t traj = i0 + q, tr_start = s_traj_row[q], tr_end = s_traj_row[q + 1];
     int64_t tu0 = s_traj_turn[q], tu1 = s_traj_turn[q + 1];
     if (r >= tr_end && q == ni - 1 && i0 + ni < p.n_traj) {
-      // past the staged trajectories (more than kScanTileRows empty ones
+      // past the staged trajectories (more than TILE empty ones
       // in the tile's rows): search the rest in global memory
       int64_t lo = i0 + ni, hi = p.n_traj - 1;
       while (lo < hi) {
@@ -428,7 +429,7 @@ __global__ void __launch_bounds__(kScanTileRows) scan_logprobs_tile_kernel(const
   // 3. segmented inclusive scan over the tile
   const TileElem tile_id = {0.0, 0.0, 0.0, 0.0, 0};
   TileElem tile_incl, tile_excl;
-  block_scan(x, tile_id, lane, warp, s_wtot, s_wpre, tile_incl, tile_excl);
+  block_scan<kWarps>(x, tile_id, lane, warp, s_wtot, s_wpre, tile_incl, tile_excl);
 
   // 4. publish the tile's aggregate, fold predecessors, publish its prefix
   if (tid == (int)(n_here - 1)) {
@@ -498,7 +499,7 @@ __global__ void __launch_bounds__(kScanTileRows) scan_logprobs_tile_kernel(const
   }
   const TrajElem traj_id = {0.0, 0, 0, 0};
   TrajElem t_incl, t_excl;
-  block_scan(te, traj_id, lane, warp, s_ttot, s_tpre, t_incl, t_excl);
+  block_scan<kWarps>(te, traj_id, lane, warp, s_ttot, s_tpre, t_incl, t_excl);
   if (live && !meta.bad) {
     stride_scan_state* sp = p.state + meta.traj;
     if (cross && (te.restart || !t_excl.crossed)) {
@@ -521,7 +522,7 @@ __global__ void __launch_bounds__(kScanTileRows) scan_logprobs_tile_kernel(const
   // the log-probs made them.
   if (!validate) return;
   bool bad = false;
-  const int64_t stride = n_tiles * kScanTileRows;
+  const int64_t stride = n_tiles * TILE;
   for (int64_t k = t0 + tid; k < p.n_turns; k += stride)
     bad |= __ldg(p.turn_row_off + k + 1) <= __ldg(p.turn_row_off + k);
   for (int64_t i = t0 + tid; i < p.n_traj; i += stride) {
@@ -565,10 +566,12 @@ cudaError_t launch_combine_partials(const float* parts, int32_t n_shards, int64_
 
 cudaError_t launch_scan_logprobs(const BatchParams& p, const float* logp_s, const float* logp_t,
                                  cudaStream_t stream, bool dependent) {
-  const int64_t n_tiles = (p.n_rows + kScanTileRows - 1) / kScanTileRows;
+  // (the small-window path's split kernel cleared the flags of its tiles)
+  const int tile_rows = dependent ? kScanTileRowsDependent : kScanTileRows;
+  const int64_t n_tiles = (p.n_rows + tile_rows - 1) / tile_rows;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3((unsigned)n_tiles);
-  cfg.blockDim = dim3(kScanTileRows);
+  cfg.blockDim = dim3((unsigned)tile_rows);
   cfg.dynamicSmemBytes = 0;
   cfg.stream = stream;
   cudaLaunchAttribute attr[1];
@@ -587,7 +590,10 @@ cudaError_t launch_scan_logprobs(const BatchParams& p, const float* logp_s, cons
   if (sms <= 0) return qe != cudaSuccess ? qe : cudaErrorInvalidDevice;
   const bool by_ticket = !dependent || n_tiles > sms;
   const cudaError_t e =
-      cudaLaunchKernelEx(&cfg, scan_logprobs_tile_kernel, p, logp_s, logp_t, n_tiles, validate, by_ticket);
+      dependent ? cudaLaunchKernelEx(&cfg, scan_logprobs_tile_kernel<kScanTileRowsDependent>, p, logp_s, logp_t,
+                                     n_tiles, validate, by_ticket)
+                : cudaLaunchKernelEx(&cfg, scan_logprobs_tile_kernel<kScanTileRows>, p, logp_s, logp_t, n_tiles,
+                                     validate, by_ticket);
   if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }
