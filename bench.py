@@ -627,12 +627,43 @@ def _graph(fn):
     return g
 
 
+def decode_compact_schedule(stride, S, T, tok, turn_end, B, ring, lam, dev):
+    """Live sets of a compacted decode sweep: run it once step by step,
+    reading each step's stop flags back (as a rollout engine does before it
+    batches the next step's live sequences).  Step s scores the live
+    rollouts' rows as rows 0..n-1 of slab s mod ring.  Returns the per-step
+    row counts and the concatenated rollout ids and turn-end flags."""
+    import torch
+
+    st = stride.new_state(B, dev)
+    sn = torch.empty(B, dtype=torch.uint8, device=dev)
+    live = np.arange(B, dtype=np.int32)
+    counts, idx, te = [], [], []
+    for s in range(turn_end.shape[0]):
+        n = live.shape[0]
+        counts.append(n)
+        if n == 0:
+            continue
+        j = s % ring
+        it = torch.from_numpy(live).to(dev)
+        tc = torch.from_numpy(np.ascontiguousarray(turn_end[s][live])).to(dev)
+        stride.stride_score_step_compact(S[j * B:j * B + n], T[j * B:j * B + n], tok[j * B:j * B + n], tc, it,
+                                         stride.TURN_MEAN, lam, st, stopped_now=sn)
+        fired = sn[:n].cpu().numpy()
+        idx.append(live.copy())
+        te.append(turn_end[s][live])
+        live = live[fired == 0]
+    return np.array(counts), np.concatenate(idx), np.concatenate(te).astype(np.uint8)
+
+
 def run_decode(args) -> None:
-    """Decode steps: B = 256 rollouts x 4,096 steps of stride_score_step, a
-    ring of 16 distinct [256, V] step slabs (more bytes than L2), turn ends
-    every U{96..768} steps, stopped rollouts masked; the 4,097 launches of a
-    sweep are replayed as one CUDA graph.  Also a 64-step graph with no stop
-    (lambda = -inf), which shows the kernel at full activity."""
+    """Decode steps: B = 256 rollouts x 4,096 steps, a ring of 16 distinct
+    [256, V] step slabs (more bytes than L2), turn ends every U{96..768}
+    steps.  Two forms of the same sweep, each replayed as one CUDA graph:
+    compacted (stride_score_step_compact over the live rollouts' rows only;
+    the reported value) and masked (stride_score_step over all 256 rows,
+    stopped rollouts masked).  Also a 64-step all-active graph (lambda =
+    -inf), which shows the kernel at full activity."""
     import torch
 
     ws, rank, local, dev = _setup_rank()
@@ -658,8 +689,25 @@ def run_decode(args) -> None:
                                      stride.TURN_MEAN, lam, st, out=out, stopped_now=sn, turn_out=tout,
                                      dev_status=status)
 
+    counts, idx_np, te_np = decode_compact_schedule(stride, S, T, tok, w["turn_end"], B, ring, w["lam_turn"], dev)
+    idx_all = torch.from_numpy(idx_np).to(dev)
+    te_all = torch.from_numpy(te_np).to(dev)
+    offs = np.concatenate([[0], np.cumsum(counts)])
+
+    def sweep_compact():
+        stride.stride_state_init(st, B)
+        for i in range(n_steps):
+            n = int(counts[i])
+            if n == 0:
+                continue
+            j, a = i % ring, int(offs[i])
+            stride.stride_score_step_compact(S[j * B:j * B + n], T[j * B:j * B + n], tok[j * B:j * B + n],
+                                             te_all[a:a + n], idx_all[a:a + n], stride.TURN_MEAN, w["lam_turn"], st,
+                                             out=out, stopped_now=sn, turn_out=tout, dev_status=status)
+
     g_full = _graph(lambda: sweep(float("-inf"), 64))
     g_run = _graph(lambda: sweep(w["lam_turn"], n_steps))
+    g_cmp = _graph(sweep_compact)
     stream = torch.cuda.current_stream()
     reps = max(1, min(args.steps, 10))
     for _ in range(max(3, args.warmup)):
@@ -669,41 +717,59 @@ def run_decode(args) -> None:
     if int(status.item()) != 0:
         raise RuntimeError(f"device status {int(status.item())}")
     scored = int(stride.state_to_numpy(st)["rows_seen"][:B].sum())
+    g_cmp.replay()
+    torch.cuda.synchronize()
+    scored_c = int(stride.state_to_numpy(st)["rows_seen"][:B].sum())
+    if int(status.item()) != 0 or scored_c != int(counts.sum()):
+        raise RuntimeError(f"compacted sweep: status {int(status.item())}, rows {scored_c} vs {int(counts.sum())}")
     a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+
+    def timed(g, n):
+        a.record(stream)
+        for _ in range(n):
+            g.replay()
+        b.record(stream)
+        torch.cuda.synchronize()
+        return a.elapsed_time(b) / n
+
     with ClockSampler(local) as clk:
         time.sleep(0.25)
-        a.record(stream)
-        for _ in range(reps):
-            g_run.replay()
-        b.record(stream)
-        torch.cuda.synchronize()
-        ms_sweep = a.elapsed_time(b) / reps
-        a.record(stream)
-        for _ in range(20):
-            g_full.replay()
-        b.record(stream)
-        torch.cuda.synchronize()
-        ms_full = a.elapsed_time(b) / 20
+        ms_cmp = timed(g_cmp, reps)
+        ms_sweep = timed(g_run, reps)
+        ms_full = timed(g_full, 20)
         time.sleep(0.05)
+    ms_cmp = max_over_ranks(ms_cmp, dev)
     ms_sweep = max_over_ranks(ms_sweep, dev)
     bpr = algorithmic_bytes_per_row(V)
     peak = measured_peaks().get("hbm_gbs", 6800.0)
     us_step_full = 1e3 * ms_full / 64
     full_gbs = B * bpr / (us_step_full * 1e-6) / 1e9
-    value = ws * scored / (ms_sweep * 1e-3)
+    cmp_gbs = scored_c * bpr / (ms_cmp * 1e-3) / 1e9
+    value = ws * scored_c / (ms_cmp * 1e-3)
+    launched = int((counts > 0).sum())
     if rank == 0:
-        line = _common_line(args, ws, ms_sweep, value)
+        line = _common_line(args, ws, ms_cmp, value)
         line.update({
             "config": {"workload": w["name"], "rollouts": B, "decode_steps": n_steps, "ring_slabs": ring,
                        "vocab": V, "stop_mode": "turn_mean", "lambda": w["lam_turn"],
-                       "tokens_scored_per_sweep": scored, "graph": "one CUDA graph per 4,097-launch sweep",
+                       "form": "compacted: each step scores only the live rollouts' rows (stride_score_step_compact)",
+                       "tokens_scored_per_sweep": scored_c, "steps_with_live_rollouts": launched,
+                       "mean_live_rollouts": float(counts.mean()),
+                       "live_rollouts_per_launched_step": {
+                           q: int(np.percentile(counts[counts > 0], float(q[1:]))) for q in ("p10", "p50", "p90")},
+                       "steps_all_live": int((counts == B).sum()),
+                       "graph": "one CUDA graph per sweep (state init + one launch per step with live rollouts)",
                        "l2": f"ring of {ring} slabs = {2 * ring * B * V * 2 / 1e9:.2f} GB > L2: no flush"},
-            "roofline": {"bound": "hbm", "achieved": full_gbs, "peak": peak, "unit": "GB/s", "frac": full_gbs / peak,
-                         "traffic": None, "kernel": "score_step_kernel<bf16,vec> (4-CTA clusters)",
-                         "us_per_step_all_active": us_step_full,
-                         "sweep_gbs_incl_masked_steps": scored * bpr / (ms_sweep * 1e-3) / 1e9,
+            "roofline": {"bound": "hbm", "achieved": cmp_gbs, "peak": peak, "unit": "GB/s", "frac": cmp_gbs / peak,
+                         "traffic": None, "kernel": "score_step_kernel<bf16,vec,compact> (cluster size from the step's rows)",
+                         "achieved_basis": "algorithmic bytes of the sweep's scored rows / sweep time",
+                         "us_per_step_all_active": us_step_full, "all_active_gbs": full_gbs,
+                         "all_active_frac": full_gbs / peak,
+                         "masked_sweep": {"ms": ms_sweep, "tokens": scored, "tokens_per_s": scored / (ms_sweep * 1e-3),
+                                          "gbs": scored * bpr / (ms_sweep * 1e-3) / 1e9,
+                                          "frac": scored * bpr / (ms_sweep * 1e-3) / 1e9 / peak},
                          "peak_source": "MEASURED_PEAKS.json hbm_gbs (of measured)"},
-            "clocks": clk.summary(), "gpu_launches": reps * (n_steps + 1) + 20 * 65,
+            "clocks": clk.summary(), "gpu_launches": reps * (launched + 1) + reps * (n_steps + 1) + 20 * 65,
         })
         print(json.dumps(line), flush=True)
 

@@ -55,10 +55,11 @@
  *   windows of at most 8 rows per SM, a kernel that splits each row over a
  *   thread-block cluster of 1, 2, 4 or 8 CTAs (the window is one wave); a
  *   persistent bulk-copy kernel for 16-byte-aligned rows; and one CTA per
- *   row otherwise.  The environment variable STRIDE_BATCH_KERNEL=split,
- *   stream or rows forces one of them, split1, split2, split4 or split8 the
- *   split kernel with that cluster size (for tests and diagnosis; stream
- *   still needs aligned rows).
+ *   row otherwise.  The decode-step calls split each row over a cluster of
+ *   1 to 16 CTAs of 128 or 512 threads, chosen from the step's row count so
+ *   that all rows run in one wave.  stride_force_batch_kernel and
+ *   stride_force_step_shape (below) fix these choices for tests and
+ *   diagnosis.
  */
 #ifndef STRIDE_H_
 #define STRIDE_H_
@@ -70,7 +71,7 @@
 extern "C" {
 #endif
 
-#define STRIDE_ABI_VERSION 2
+#define STRIDE_ABI_VERSION 3
 
 #if defined(__GNUC__)
 #define STRIDE_API __attribute__((visibility("default")))
@@ -293,6 +294,33 @@ STRIDE_API int stride_score_step(const void* S, const void* T, int32_t dtype, in
                       uint8_t* stopped_now, stride_turn_stats* turn_out, int32_t* dev_status,
                       void* stream);
 
+/* stride_score_step with the live rollouts' rows packed (Algorithm 1, inner
+ * turn loop: only rollouts that have not stopped generate a token, so a
+ * rollout engine that batches only live sequences hands over one row per
+ * live rollout).
+ *
+ * Row b (0 <= b < n_rows) of S, T ([n_rows, ld]), tokens (int32 [n_rows]),
+ * turn_end (uint8 [n_rows]) and of every per-row output (out, stopped_now,
+ * turn_out: [n_rows] each, nullable) belongs to rollout rollout_idx[b]
+ * (device int32 [n_rows], distinct values in [0, n_rollouts)), whose carried
+ * state is state[rollout_idx[b]] (device [n_rollouts], in/out) and whose
+ * threshold is lambda[rollout_idx[b]] (device float [n_rollouts]) or
+ * lambda_all.  The step rule is that of stride_score_step.  Unlike the
+ * masked form, a row's logits are read before its state: a row whose
+ * rollout has already stopped is read, not scored (NaN outputs, state
+ * unchanged).  An index outside [0, n_rollouts) sets STRIDE_DEV_BAD_LAYOUT
+ * and NaN outputs for that row; repeated indices race.  The cluster size
+ * grows as n_rows shrinks, so a step of a few live rollouts still spreads
+ * its rows over the GPU.  No workspace; n_rows = 0 launches nothing. */
+STRIDE_API int stride_score_step_compact(const void* S, const void* T, int32_t dtype, int64_t ld,
+                                         int64_t V, const int32_t* tokens, const uint8_t* turn_end,
+                                         const int32_t* rollout_idx, int32_t n_rows,
+                                         int32_t n_rollouts, int32_t stop_mode, const float* lambda,
+                                         float lambda_all, stride_scan_state* state,
+                                         const stride_row_outputs* out, uint8_t* stopped_now,
+                                         stride_turn_stats* turn_out, int32_t* dev_status,
+                                         void* stream);
+
 /* Restart choice over N stored trajectory records (Sec. 4.2 steps 1-2,
  * Eq. 6, Algorithm 1).
  *
@@ -362,6 +390,25 @@ STRIDE_API int stride_buffer_record(float* buf_mean, int32_t* buf_n_turns, int32
                                     const int32_t* k0_of_traj, const stride_turn_stats* turn_stats,
                                     const int32_t* traj_turn_off, int32_t n_traj,
                                     int32_t* dev_status, void* stream);
+
+/* ---- diagnostic overrides (no counterpart in the paper) ----------------------
+ * Process-wide settings for tests and diagnosis; they change which kernel
+ * runs, never the results beyond floating-point rounding.  Set them between
+ * calls, not while other threads launch.
+ *
+ * stride_force_batch_kernel: NULL, "" or "auto" = automatic choice; "split"
+ * (automatic cluster size), "split1", "split2", "split4", "split8" (the
+ * small-window kernel with that cluster size), "stream" (the persistent
+ * kernel; rows that are not 16-byte aligned still take the per-row kernel)
+ * or "rows" (one CTA per row).  Its initial value is the environment variable
+ * STRIDE_BATCH_KERNEL (same names), read once, at the first batch call.
+ * stride_force_step_shape: the decode-step calls' CTA size (128 or 512
+ * threads; 0 = 128 when a cluster size is given) and CTAs per row (1..16;
+ * 0 = 1 when a CTA size is given); (0, 0) = automatic.  A shape the device
+ * cannot place makes the step calls return STRIDE_ERR_CUDA.
+ * Both return STRIDE_ERR_INVALID_ARG for an unknown name, size or shape. */
+STRIDE_API int stride_force_batch_kernel(const char* name);
+STRIDE_API int stride_force_step_shape(int32_t cta_threads, int32_t cluster_size);
 
 /* Human-readable name of a stride_status code (static string). */
 STRIDE_API const char* stride_status_string(int code);

@@ -217,8 +217,13 @@ class Rollouts(ctypes.Structure):
 
 
 def rollouts_to_numpy(state) -> dict:
-    keys = [f[0] for f in Rollouts._fields_]
-    return {k: np.array([getattr(s, k) for s in state]) for k in keys}
+    v = rollouts_view(state)
+    return {k: v[k].copy() for k in v.dtype.names}
+
+
+def rollouts_view(state) -> np.ndarray:
+    """A live numpy structured view of a rollout array (no copy)."""
+    return np.frombuffer(state, dtype=np.dtype(Rollouts))
 
 
 def _ptr(a):

@@ -80,6 +80,10 @@ def lib() -> ctypes.CDLL:
         L.stride_score_batch.argtypes = [P, P, i32, i64, i64, P, P, P, P, i32, i32, i64, i64, i32, P, f32,
                                          P, P, P, P, P, P, sz, P]
         L.stride_score_step.argtypes = [P, P, i32, i64, i64, P, P, i32, i32, P, f32, P, P, P, P, P, P]
+        L.stride_score_step_compact.argtypes = [P, P, i32, i64, i64, P, P, P, i32, i32, i32, P, f32, P, P, P, P,
+                                                P, P]
+        L.stride_force_batch_kernel.argtypes = [ctypes.c_char_p]
+        L.stride_force_step_shape.argtypes = [i32, i32]
         L.stride_select_restart.argtypes = [P, P, P, f32, i32, i32, P, P, P]
         L.stride_buffer_record.argtypes = [P, P, i32, i32, P, P, P, P, i32, P, P]
         L.stride_partial_lse.argtypes = [P, P, i32, i64, i64, i64, P, i64, P, P, P]
@@ -99,7 +103,8 @@ def lib() -> ctypes.CDLL:
         L.stride_status_string.restype = ctypes.c_char_p
         L.stride_abi_version.restype = ctypes.c_int
         for fn in ("stride_state_init", "stride_score_batch", "stride_score_step", "stride_select_restart",
-                   "stride_score_batch_noalloc"):
+                   "stride_score_batch_noalloc", "stride_score_step_compact", "stride_force_batch_kernel",
+                   "stride_force_step_shape"):
             getattr(L, fn).restype = ctypes.c_int
         _LIB = L
     return _LIB
@@ -283,6 +288,42 @@ def stride_score_step(S, T, tokens, turn_end, stop_mode: int, lam, state, out: d
         _dev(turn_out, "turn_out", torch.uint8, B * TURN_STATS_DTYPE.itemsize, optional=True),
         _dev(dev_status, "dev_status", torch.int32, 1, optional=True), _stream(stream))
     _check("stride_score_step", rc)
+
+
+def stride_score_step_compact(S, T, tokens, turn_end, rollout_idx, stop_mode: int, lam, state,
+                              out: dict | None = None, stopped_now=None, turn_out=None, dev_status=None,
+                              V: int | None = None, n_rows: int | None = None, stream=None) -> None:
+    """One decode step over the live rollouts, their rows packed: row b of
+    S, T, tokens, turn_end and the outputs is rollout rollout_idx[b] (int32
+    CUDA tensor of n_rows = len(rollout_idx) entries unless given) of the
+    state tensor's rollouts (see include/stride.h)."""
+    torch = _torch()
+    dt, ld = _logits(S, T)
+    n = int(rollout_idx.shape[0]) if n_rows is None else int(n_rows)
+    if n > S.shape[0]:
+        raise ValueError("S and T need a row per live rollout")
+    n_state = state.numel() // STATE_DTYPE.itemsize
+    V = S.shape[1] if V is None else int(V)
+    lam_p, lam_all = _lambda(lam, n_state)
+    rc = lib().stride_score_step_compact(
+        S.data_ptr(), T.data_ptr(), dt, ld, V, _dev(tokens, "tokens", torch.int32, n),
+        _dev(turn_end, "turn_end", torch.uint8, n), _dev(rollout_idx, "rollout_idx", torch.int32, n), n, n_state,
+        int(stop_mode), lam_p, lam_all, _dev(state, "state", torch.uint8, n_state * STATE_DTYPE.itemsize),
+        _row_outputs(out, n), _dev(stopped_now, "stopped_now", torch.uint8, n, optional=True),
+        _dev(turn_out, "turn_out", torch.uint8, n * TURN_STATS_DTYPE.itemsize, optional=True),
+        _dev(dev_status, "dev_status", torch.int32, 1, optional=True), _stream(stream))
+    _check("stride_score_step_compact", rc)
+
+
+def stride_force_batch_kernel(name: str | None) -> None:
+    """Fix the batch kernel for tests and diagnosis (None / "auto": automatic)."""
+    _check("stride_force_batch_kernel", lib().stride_force_batch_kernel(None if name is None else name.encode()))
+
+
+def stride_force_step_shape(cta_threads: int, cluster_size: int) -> None:
+    """Fix the decode step's CTA size (128 or 512) and CTAs per row for tests
+    and diagnosis ((0, 0): automatic)."""
+    _check("stride_force_step_shape", lib().stride_force_step_shape(int(cta_threads), int(cluster_size)))
 
 
 def stride_select_restart(turn_mean, n_turns, correct, alpha: float, k_star, k_max, stream=None) -> None:

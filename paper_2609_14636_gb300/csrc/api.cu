@@ -224,20 +224,25 @@ int stride_score_batch_multi_teacher(const void* S, const void* const* T_domains
                                                                                      : STRIDE_ERR_CUDA;
 }
 
-int stride_score_step(const void* S, const void* T, int32_t dtype, int64_t ld, int64_t V,
-                      const int32_t* tokens, const uint8_t* turn_end, int32_t B,
-                      int32_t stop_mode, const float* lambda, float lambda_all,
-                      stride_scan_state* state, const stride_row_outputs* out,
+}  // extern "C"
+
+namespace {
+
+// Checks and launch shared by the two decode-step entry points.
+int score_step_common(const void* S, const void* T, int32_t dtype, int64_t ld, int64_t V,
+                      const int32_t* tokens, const uint8_t* turn_end, const int32_t* rollout_idx,
+                      int32_t rows, int32_t n_state, int32_t stop_mode, const float* lambda,
+                      float lambda_all, stride_scan_state* state, const stride_row_outputs* out,
                       uint8_t* stopped_now, stride_turn_stats* turn_out, int32_t* dev_status,
                       void* stream) {
   const int lc = check_logits(S, T, dtype, ld, V);
   if (lc != STRIDE_OK) return lc;
-  if (B < 0 || B > (INT32_MAX / 8)) return STRIDE_ERR_INVALID_ARG;
+  if (rows < 0 || rows > (INT32_MAX / 16) || n_state < 0) return STRIDE_ERR_INVALID_ARG;
   if (stop_mode != STRIDE_STOP_TURN_MEAN && stop_mode != STRIDE_STOP_TOKEN_SUM)
     return STRIDE_ERR_INVALID_ARG;
   if (!lambda && isnan(lambda_all)) return STRIDE_ERR_INVALID_ARG;
-  if (B == 0) return STRIDE_OK;
-  if (!tokens || !turn_end || !state) return STRIDE_ERR_INVALID_ARG;
+  if (rows == 0) return STRIDE_OK;
+  if (!tokens || !turn_end || !state || n_state < 1) return STRIDE_ERR_INVALID_ARG;
   const int dc = check_device();
   if (dc != STRIDE_OK) return dc;
   stride::StepParams p;
@@ -248,7 +253,9 @@ int stride_score_step(const void* S, const void* T, int32_t dtype, int64_t ld, i
   p.mode = stop_mode;
   p.tokens = tokens;
   p.turn_end = turn_end;
-  p.B = B;
+  p.rollout_idx = rollout_idx;
+  p.B = rows;
+  p.n_state = n_state;
   p.lambda = lambda;
   p.lambda_all = lambda_all;
   p.state = state;
@@ -260,6 +267,41 @@ int stride_score_step(const void* S, const void* T, int32_t dtype, int64_t ld, i
   return stride::launch_score_step(p, dtype, vec, (cudaStream_t)stream) == cudaSuccess
              ? STRIDE_OK
              : STRIDE_ERR_CUDA;
+}
+
+}  // namespace
+
+extern "C" {
+
+int stride_score_step(const void* S, const void* T, int32_t dtype, int64_t ld, int64_t V,
+                      const int32_t* tokens, const uint8_t* turn_end, int32_t B,
+                      int32_t stop_mode, const float* lambda, float lambda_all,
+                      stride_scan_state* state, const stride_row_outputs* out,
+                      uint8_t* stopped_now, stride_turn_stats* turn_out, int32_t* dev_status,
+                      void* stream) {
+  return score_step_common(S, T, dtype, ld, V, tokens, turn_end, nullptr, B, B, stop_mode, lambda,
+                           lambda_all, state, out, stopped_now, turn_out, dev_status, stream);
+}
+
+int stride_score_step_compact(const void* S, const void* T, int32_t dtype, int64_t ld, int64_t V,
+                              const int32_t* tokens, const uint8_t* turn_end,
+                              const int32_t* rollout_idx, int32_t n_rows, int32_t n_rollouts,
+                              int32_t stop_mode, const float* lambda, float lambda_all,
+                              stride_scan_state* state, const stride_row_outputs* out,
+                              uint8_t* stopped_now, stride_turn_stats* turn_out,
+                              int32_t* dev_status, void* stream) {
+  if (n_rows > 0 && !rollout_idx) return STRIDE_ERR_INVALID_ARG;
+  return score_step_common(S, T, dtype, ld, V, tokens, turn_end, rollout_idx, n_rows, n_rollouts,
+                           stop_mode, lambda, lambda_all, state, out, stopped_now, turn_out,
+                           dev_status, stream);
+}
+
+int stride_force_batch_kernel(const char* name) {
+  return stride::set_batch_kernel_override(name) == 0 ? STRIDE_OK : STRIDE_ERR_INVALID_ARG;
+}
+
+int stride_force_step_shape(int32_t cta_threads, int32_t cluster_size) {
+  return stride::set_step_shape_override(cta_threads, cluster_size) == 0 ? STRIDE_OK : STRIDE_ERR_INVALID_ARG;
 }
 
 int stride_select_restart(const float* turn_mean, const int32_t* n_turns, const uint8_t* correct,

@@ -21,6 +21,7 @@
 #include <string.h>
 
 #include <atomic>
+#include <mutex>
 
 #include "stride.h"
 #include "stride_device.cuh"
@@ -307,6 +308,46 @@ static int split_cluster(int64_t n_rows, int sms) {
   return 0;
 }
 
+// Forced batch kernel (tests and diagnosis): 0 automatic, kForceStream,
+// kForceRows, or kForceSplit + C (C = 0: the split kernel with its automatic
+// cluster size).  Its first value comes from the environment variable
+// STRIDE_BATCH_KERNEL, read once per process at the first batch call;
+// stride_force_batch_kernel changes it.
+constexpr int kForceStream = 1, kForceRows = 2, kForceSplit = 16;
+static std::atomic<int> g_batch_force{-1};  // -1: environment not read yet
+
+static int parse_batch_kernel(const char* name) {
+  if (!name || !*name || !strcmp(name, "auto")) return 0;
+  if (!strcmp(name, "stream")) return kForceStream;
+  if (!strcmp(name, "rows")) return kForceRows;
+  if (!strcmp(name, "split")) return kForceSplit;
+  if (!strcmp(name, "split1")) return kForceSplit + 1;
+  if (!strcmp(name, "split2")) return kForceSplit + 2;
+  if (!strcmp(name, "split4")) return kForceSplit + 4;
+  if (!strcmp(name, "split8")) return kForceSplit + 8;
+  return -1;
+}
+
+static int batch_kernel_override() {
+  int f = g_batch_force.load(std::memory_order_relaxed);
+  if (f >= 0) return f;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    const int v = parse_batch_kernel(getenv("STRIDE_BATCH_KERNEL"));
+    int expect = -1;
+    g_batch_force.compare_exchange_strong(expect, v < 0 ? 0 : v);
+  });
+  return g_batch_force.load(std::memory_order_relaxed);
+}
+
+int set_batch_kernel_override(const char* name) {
+  const int v = parse_batch_kernel(name);
+  if (v < 0) return -1;
+  (void)batch_kernel_override();  // the environment's value, if any, is superseded from here on
+  g_batch_force.store(v, std::memory_order_relaxed);
+  return 0;
+}
+
 template <typename LT, bool VEC>
 static cudaError_t launch_split(const BatchParams& p, int C, cudaStream_t stream) {
   cudaLaunchConfig_t cfg = {};
@@ -335,18 +376,14 @@ cudaError_t launch_score_batch(const BatchParams& p, int dtype, bool vec, size_t
   cudaError_t qe = cudaSuccess;
   const int sms = current_device_sms(&dev, &qe);
   if (sms <= 0) return qe != cudaSuccess ? qe : cudaErrorInvalidDevice;
-  // STRIDE_BATCH_KERNEL = split | split1 | split2 | split4 | split8 |
-  // stream | rows forces one kernel, or the split kernel with one cluster
-  // size (tests and diagnosis); anything else, or unset, chooses by window
-  // size.
-  const char* force = getenv("STRIDE_BATCH_KERNEL");
-  const bool f_split = force && !strncmp(force, "split", 5);
-  const bool f_stream = force && !strcmp(force, "stream");
-  const bool f_rows = force && !strcmp(force, "rows");
+  const int force = batch_kernel_override();
+  const bool f_split = force >= kForceSplit;
+  const bool f_stream = force == kForceStream;
+  const bool f_rows = force == kForceRows;
   int C = (f_stream || f_rows) ? 0 : split_cluster(p.n_rows, sms);
   if (f_split) {
-    const int want = atoi(force + 5);
-    if (want == 1 || want == 2 || want == 4 || want == 8) C = want;
+    const int want = force - kForceSplit;
+    if (want > 0) C = want;
     else if (C == 0) C = 2;
   }
   if (C > 0 && p.V < 32 * (int64_t)C) C = f_split ? 1 : 0;  // a few logits per rank at least

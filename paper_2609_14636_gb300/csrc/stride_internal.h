@@ -83,7 +83,9 @@ struct StepParams {
   int32_t mode;
   const int32_t* tokens;
   const uint8_t* turn_end;
-  int32_t B;
+  const int32_t* rollout_idx;  // compacted rows: row b is rollout rollout_idx[b]; NULL = row b is rollout b
+  int32_t B;                   // rows of this step
+  int32_t n_state;             // rollouts in state / lambda (compacted form: bound of rollout_idx)
   const float* lambda;
   float lambda_all;
   stride_scan_state* state;
@@ -139,6 +141,10 @@ int current_device_sms(int* dev_out, cudaError_t* err);
 cudaError_t launch_score_batch(const BatchParams& p, int dtype, bool vec, size_t clear_bytes, cudaStream_t stream);
 cudaError_t launch_score_batch_stream(const BatchParams& p, int dtype, cudaStream_t stream);
 cudaError_t launch_score_step(const StepParams& p, int dtype, bool vec, cudaStream_t stream);
+// Diagnostic overrides of the automatic kernel choices (process-wide; 0 on
+// success, -1 for a value out of range).
+int set_step_shape_override(int threads, int C);  // 0 = automatic; 128 or 512 threads, 1..16 CTAs per row
+int set_batch_kernel_override(const char* name);  // NULL / "" / "auto" = automatic
 cudaError_t launch_select_restart(const SelectParams& p, cudaStream_t stream);
 cudaError_t launch_state_init(stride_scan_state* state, int32_t n, cudaStream_t stream);
 cudaError_t launch_partial_lse(const void* S, const void* T, int dtype, bool vec, int64_t ld,

@@ -37,7 +37,7 @@ def test_library_exports_declared_symbols():
 def test_host_only_calls():
     import paper_2609_14636_gb300 as stride
 
-    assert stride.stride_abi_version() == 2
+    assert stride.stride_abi_version() == 3
     assert stride.stride_score_batch_workspace_size(0) == 0
     assert stride.stride_score_batch_workspace_size(1000) >= 1000 * 68
     assert "INVALID_ARG" in stride.stride_status_string(1)

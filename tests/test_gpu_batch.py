@@ -23,15 +23,13 @@ def stride():
 
 
 @pytest.fixture(params=["auto", "stream", "split", "split1", "split8", "rows"])
-def kernel(request, monkeypatch):
+def kernel(request, stride):
     """Runs a test under each of the batch kernels, and the split kernel at
     its automatic, smallest (one CTA per row) and largest (8-CTA) cluster
-    size (the library reads STRIDE_BATCH_KERNEL on every call)."""
-    if request.param == "auto":
-        monkeypatch.delenv("STRIDE_BATCH_KERNEL", raising=False)
-    else:
-        monkeypatch.setenv("STRIDE_BATCH_KERNEL", request.param)
-    return request.param
+    size (stride_force_batch_kernel; automatic again afterwards)."""
+    stride.stride_force_batch_kernel(request.param)
+    yield request.param
+    stride.stride_force_batch_kernel("auto")
 
 
 def _bf16_rows(seed, R, V, sigma=4.0, noise=0.5):
