@@ -31,12 +31,12 @@
  *                         longest correct prefix K_max and the weakest correct
  *                         turn k* of Eq. 6 (Algorithm 1, K_max / k* / K0).
  *
- * Readings where the paper is silent (each is also listed in the design
- * notes): sums are strict "< lambda" and "> alpha"; turns are 0-based, so the
- * returned k* equals K0 (the number of reused turns); ties in Eq. 6 go to the
- * lowest index; K_max = 0 gives k* = 0; an empty turn is an error; a row whose
- * logits are all -inf has LSE = -inf and NaN log-probs; an out-of-range token
- * gives NaN for its row and an error return.
+ * Readings where the paper is silent: sums are strict "< lambda" and
+ * "> alpha"; turns are 0-based, so the returned k* equals K0 (the number of
+ * reused turns); ties in Eq. 6 go to the lowest index; K_max = 0 gives
+ * k* = 0; an empty turn is an error; a row whose logits are all -inf has
+ * LSE = -inf and NaN log-probs; an out-of-range token gives NaN for its row
+ * and an error return.
  *
  * Parity pins: see tests/test_oracle_pins.py (closed forms, brute force in
  * arbitrary precision, invariants, hand-worked cases in tests/golden/).
