@@ -20,9 +20,12 @@
 //   cudaMemsetAsync, or from the small-window kernel).  Two calls that
 //   overlap in time on the GPU race on the array and give wrong results:
 //   order them on one stream (or with events);
-// - the first call on a device looks up the array's device address with
-//   cudaGetSymbolAddress (this may load the library's module onto the
-//   device); make that first call before any stream capture.
+// - the array's device address comes from cudaGetSymbolAddress (the first
+//   call on a device may load the library's module onto it, so make that
+//   first call before any stream capture).  It is looked up again on every
+//   call made outside a stream capture, so a device reset between calls
+//   (which may move the array) is followed; a call made while its stream is
+//   capturing uses the address the last such call found.
 // Nothing here calls cudaMalloc, cudaFree or any allocating routine.
 #include <cuda_runtime.h>
 #include <math.h>
@@ -53,14 +56,18 @@ constexpr int kMaxDevices = 64;
 void* g_scratch_addr[kMaxDevices] = {};
 std::mutex g_setup_mutex;
 
-// Device address of the scratch on the current device, looked up once per
-// device (with that device current).
-int scratch_for_current_device(void** out) {
+// Device address of the scratch on the current device (with that device
+// current): looked up afresh unless `stream` is capturing, in which case the
+// address found by the last lookup on this device is used.
+int scratch_for_current_device(cudaStream_t stream, void** out) {
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess) return STRIDE_ERR_CUDA;
   if (dev < 0 || dev >= kMaxDevices) return STRIDE_ERR_UNSUPPORTED_DEVICE;
+  cudaStreamCaptureStatus cap = cudaStreamCaptureStatusNone;
+  if (cudaStreamIsCapturing(stream, &cap) != cudaSuccess) return STRIDE_ERR_CUDA;
   std::lock_guard<std::mutex> lock(g_setup_mutex);
-  if (g_scratch_addr[dev] == nullptr) {
+  if (cap == cudaStreamCaptureStatusNone || g_scratch_addr[dev] == nullptr) {
+    if (cap != cudaStreamCaptureStatusNone) return STRIDE_ERR_CUDA;  // no address found before the capture
     void* ptr = nullptr;
     if (cudaGetSymbolAddress(&ptr, g_noalloc_scratch) != cudaSuccess || ptr == nullptr)
       return STRIDE_ERR_CUDA;
@@ -80,12 +87,15 @@ extern "C" STRIDE_API int stride_score_batch_noalloc(
     stride_turn_stats* turn_stats, double* profile, int32_t* dev_status, void* stream) {
   if (row_begin < 0 || row_end < row_begin) return STRIDE_ERR_INVALID_ARG;
   if (row_end - row_begin > (int64_t)STRIDE_NOALLOC_MAX_ROWS) return STRIDE_ERR_TOO_LARGE;
-  if (row_end == row_begin) return STRIDE_OK;
+  if (row_end == row_begin)  // the same argument checks as the workspace entry point, nothing launched
+    return stride_score_batch(S, T, dtype, ld, V, tokens, traj_row_off, turn_row_off, traj_turn_off,
+                              n_traj, n_turns, row_begin, row_end, stop_mode, lambda, lambda_all, state,
+                              out, turn_stats, profile, dev_status, nullptr, 0, stream);
   static_assert(kNoAllocBytes % 256 == 0, "scratch size");
   if (stride::batch_workspace_layout(STRIDE_NOALLOC_MAX_ROWS).total > kNoAllocBytes)
     return STRIDE_ERR_CUDA;  // layout and array out of step: a build error, never expected
   void* scratch = nullptr;
-  const int sc = scratch_for_current_device(&scratch);
+  const int sc = scratch_for_current_device((cudaStream_t)stream, &scratch);
   if (sc != STRIDE_OK) return sc;
   // The scoring entry point clears the tickets and flags of the window and
   // launches the kernels with pointers into the scratch.

@@ -114,3 +114,33 @@ def test_noalloc_rejects_oversize_window():
     torch.cuda.synchronize()
     assert int(status.item()) == 0
     assert np.allclose(out["logp_t"].cpu().numpy(), -np.log(8.0), atol=LOGP_ATOL)
+
+
+def test_noalloc_empty_window_checks_arguments():
+    """An empty window launches nothing but gets the workspace entry point's
+    argument checks: a bad stop mode, no trajectories or missing offsets are
+    rejected by both entry points alike."""
+    import torch
+
+    import paper_2609_14636_gb300 as stride
+
+    lay = synth.layout_from_turn_lengths([[4, 3]])
+    S = torch.zeros((lay.rows, 8), dtype=torch.bfloat16, device="cuda")
+    tk = torch.zeros(lay.rows, dtype=torch.int32, device="cuda")
+    offs = [torch.from_numpy(a).cuda().data_ptr() for a in (lay.traj_row_off, lay.turn_row_off, lay.traj_turn_off)]
+    st = stride.new_state(1)
+    L = stride.lib()
+
+    def both(mode, n_traj, offsets):
+        a = L.stride_score_batch(S.data_ptr(), S.data_ptr(), 0, 8, 8, tk.data_ptr(), *offsets, n_traj,
+                                 lay.n_turns, 2, 2, mode, None, -1.0, st.data_ptr(), None, None, None, None,
+                                 None, 0, None)
+        b = L.stride_score_batch_noalloc(S.data_ptr(), S.data_ptr(), 0, 8, 8, tk.data_ptr(), *offsets, n_traj,
+                                         lay.n_turns, 2, 2, mode, None, -1.0, st.data_ptr(), None, None, None,
+                                         None, None)
+        return a, b
+
+    assert both(0, 1, offs) == (stride.OK, stride.OK)
+    assert both(7, 1, offs) == (stride.ERR_INVALID_ARG, stride.ERR_INVALID_ARG)
+    assert both(0, 0, offs) == (stride.ERR_INVALID_ARG, stride.ERR_INVALID_ARG)
+    assert both(0, 1, [offs[0], None, offs[2]]) == (stride.ERR_INVALID_ARG, stride.ERR_INVALID_ARG)
