@@ -357,9 +357,14 @@ STRIDE_API int stride_select_restart(const float* turn_mean, const int32_t* n_tu
  * - All calls on a device share the one scratch array, which keeps the last
  *   call's contents; each call clears what must start at zero.  Calls that
  *   overlap in time on the GPU race on it: order them on one stream.
- * - The first call on a device looks up the array's device address
- *   (cudaGetSymbolAddress, once per device); make that first call before any
- *   stream capture. */
+ * - The array's device address is looked up (cudaGetSymbolAddress) on every
+ *   call made outside a stream capture, so a device reset between calls is
+ *   followed; the first call on a device may load the library's module, so
+ *   make it before any stream capture.  A call on a capturing stream uses
+ *   the address found by the last call outside a capture (none yet:
+ *   STRIDE_ERR_CUDA).
+ * - An empty window (row_begin == row_end) gets the argument checks of
+ *   stride_score_batch and launches nothing. */
 #define STRIDE_NOALLOC_MAX_ROWS 65536
 STRIDE_API int stride_score_batch_noalloc(const void* S, const void* T, int32_t dtype, int64_t ld,
                                           int64_t V, const int32_t* tokens,

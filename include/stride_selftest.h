@@ -1,9 +1,13 @@
 /*
- * stride_selftest.h -- a self-test hook for the bounded device-side waits of
- * libstride.so.  The paper has no counterpart: this exists so that the
- * library's failure path (a wait that runs out sets STRIDE_DEV_TIMEOUT and
- * the kernel returns, leaving the context usable) can be exercised on a GPU
- * without faulting or hanging it.
+ * stride_selftest.h -- self-test and measurement hooks of libstride.so.  The
+ * paper has no counterpart to either:
+ * - the bounded-wait self-test exists so that the library's failure path (a
+ *   wait that runs out sets STRIDE_DEV_TIMEOUT and the kernel returns,
+ *   leaving the context usable) can be exercised on a GPU without faulting
+ *   or hanging it;
+ * - the read-only stream gives the floor the scoring kernels are measured
+ *   against: how fast this GPU reads the same bytes, in the same 16-byte
+ *   loads, with no arithmetic at all.
  */
 #ifndef STRIDE_SELFTEST_H_
 #define STRIDE_SELFTEST_H_
@@ -26,6 +30,17 @@ extern "C" {
  * STRIDE_OK after the launch, or an argument / CUDA error code. */
 STRIDE_API int stride_selftest_bounded_wait(int32_t which, uint64_t timeout_ns, int32_t* dev_status,
                                             void* workspace, size_t workspace_bytes, void* stream);
+
+/* Reads bytes_each bytes of device buffer a, and of b when b is not NULL,
+ * once, with the scoring kernels' 16-byte non-allocating loads: `grid` CTAs
+ * of `threads` threads (a multiple of 32, at most 1,024), CTA c reading the
+ * c-th contiguous 1/grid of each buffer.  Nothing is computed beyond an XOR
+ * of the loaded words, written as one word per CTA to sink (device uint32
+ * [grid]) so the loads cannot be dropped.  a and b must be 16-byte aligned
+ * and bytes_each a multiple of 16.  Asynchronous on stream; returns STRIDE_OK
+ * after the launch, or an argument / CUDA error code. */
+STRIDE_API int stride_selftest_stream_read(const void* a, const void* b, uint64_t bytes_each, int32_t grid,
+                                           int32_t threads, uint32_t* sink, void* stream);
 
 #ifdef __cplusplus
 }

@@ -28,7 +28,9 @@ __all__ = [
     "new_turn_stats", "state_to_numpy", "turn_stats_to_numpy", "stride_state_init",
     "stride_score_batch_workspace_size", "stride_score_batch", "stride_score_step",
     "stride_select_restart", "stride_status_string", "stride_abi_version", "ROW_OUTPUT_KEYS",
-    "stride_score_batch_noalloc", "NOALLOC_MAX_ROWS", "ERR_TOO_LARGE", "PROFILE_BINS", "new_profile",
+    "stride_score_batch_noalloc", "NOALLOC_MAX_ROWS", "OK", "ERR_INVALID_ARG", "ERR_UNSUPPORTED_DTYPE",
+    "ERR_WORKSPACE", "ERR_CUDA", "ERR_UNSUPPORTED_DEVICE", "ERR_TOO_LARGE", "PROFILE_BINS", "new_profile",
+    "stride_score_step_compact", "stride_force_batch_kernel", "stride_force_step_shape",
     "stride_selftest_bounded_wait", "stride_buffer_record", "stride_score_batch_multi_teacher",
     "multi_teacher_workspace_size", "stride_partial_lse", "stride_combine_partials", "stride_scan_logprobs",
 ]
@@ -38,7 +40,7 @@ TURN_MEAN, TOKEN_SUM = 0, 1
 DEV_TOKEN_RANGE, DEV_BAD_LAYOUT, DEV_TIMEOUT = 0x1, 0x2, 0x4
 ROW_OUTPUT_KEYS = ("logp_s", "logp_t", "opd", "lse_s", "lse_t", "x_s", "x_t")
 NOALLOC_MAX_ROWS = 65536  # STRIDE_NOALLOC_MAX_ROWS
-ERR_TOO_LARGE = 6
+OK, ERR_INVALID_ARG, ERR_UNSUPPORTED_DTYPE, ERR_WORKSPACE, ERR_CUDA, ERR_UNSUPPORTED_DEVICE, ERR_TOO_LARGE = range(7)
 
 STATE_DTYPE = np.dtype([("cum", "<f8"), ("turn_sum_t", "<f8"), ("turn_sum_d", "<f8"),
                         ("turn_sum_l", "<f8"), ("loss", "<f8"), ("rows_seen", "<i8"),
@@ -97,6 +99,8 @@ def lib() -> ctypes.CDLL:
         L.stride_buffer_record.restype = ctypes.c_int
         L.stride_selftest_bounded_wait.argtypes = [i32, ctypes.c_uint64, P, P, sz, P]
         L.stride_selftest_bounded_wait.restype = ctypes.c_int
+        L.stride_selftest_stream_read.argtypes = [P, P, ctypes.c_uint64, i32, i32, P, P]
+        L.stride_selftest_stream_read.restype = ctypes.c_int
         L.stride_score_batch_noalloc.argtypes = [P, P, i32, i64, i64, P, P, P, P, i32, i32, i64, i64, i32,
                                                  P, f32, P, P, P, P, P, P]
         L.stride_status_string.argtypes = [ctypes.c_int]
@@ -474,6 +478,20 @@ def stride_selftest_bounded_wait(which: int, timeout_ns: int, dev_status, worksp
     rc = lib().stride_selftest_bounded_wait(int(which), int(timeout_ns), _dev(dev_status, "dev_status", torch.int32, 1),
                                             _dev(workspace, "workspace", torch.uint8), workspace.numel(), _stream(stream))
     _check("stride_selftest_bounded_wait", rc)
+
+
+def stride_selftest_stream_read(a, b, bytes_each: int, grid: int, threads: int, sink, stream=None) -> None:
+    """Read-only stream over bytes_each bytes of CUDA tensors a (and b, or
+    None) with the scoring kernels' loads (see include/stride_selftest.h)."""
+    torch = _torch()
+    for name, x in (("a", a), ("b", b)):
+        if x is not None and (not isinstance(x, torch.Tensor) or not x.is_cuda or not x.is_contiguous()
+                              or x.numel() * x.element_size() < bytes_each):
+            raise ValueError(f"{name} must be a contiguous CUDA tensor of at least {bytes_each} bytes")
+    rc = lib().stride_selftest_stream_read(a.data_ptr(), None if b is None else b.data_ptr(), int(bytes_each),
+                                           int(grid), int(threads), _dev(sink, "sink", torch.int32, int(grid)),
+                                           _stream(stream))
+    _check("stride_selftest_stream_read", rc)
 
 
 def stride_score_batch_noalloc(S, T, tokens, traj_row_off, turn_row_off, traj_turn_off, row_begin: int,

@@ -1,10 +1,14 @@
-// selftest.cu -- runs the library's real bounded waits on a flag (or an
-// mbarrier) that nothing sets, so that the timeout path can be checked on a
-// GPU: the wait runs out after timeout_ns, the kernel records
-// STRIDE_DEV_TIMEOUT and returns.  No trap, no fault, no endless loop.
+// selftest.cu -- two hooks that are not part of the scoring path:
+// * the library's real bounded waits run on a flag (or an mbarrier) that
+//   nothing sets, so that the timeout path can be checked on a GPU: the wait
+//   runs out after timeout_ns, the kernel records STRIDE_DEV_TIMEOUT and
+//   returns.  No trap, no fault, no endless loop;
+// * a read-only stream over one or two buffers, the floor the scoring
+//   kernels are measured against.
 #include <cuda_runtime.h>
 
 #include "mbarrier.cuh"
+#include "stride_device.cuh"
 #include "row_scan.cuh"
 #include "stride.h"
 #include "stride_internal.h"
@@ -34,7 +38,65 @@ __global__ void selftest_mbarrier_kernel(int32_t* dev_status, uint64_t timeout_n
   if (threadIdx.x == 0 && !ok) set_status(dev_status, STRIDE_DEV_TIMEOUT);
 }
 
+// Read-only streaming: CTA c reads its contiguous 1/grid of the 16-byte
+// vectors of a (and of b), with the scoring kernels' non-allocating 16-byte
+// loads, 8 in flight per thread per buffer, and folds them with XOR so the
+// loads stay live; one word per CTA is written to sink.
+__global__ void stream_read_kernel(const uint4* __restrict__ a, const uint4* __restrict__ b, uint64_t nv,
+                                   uint32_t* __restrict__ sink) {
+  const uint64_t g = gridDim.x;
+  const uint64_t lo = nv * blockIdx.x / g, hi = nv * (blockIdx.x + 1) / g;
+  constexpr int U = 8;
+  uint32_t x = 0;
+  uint64_t i = lo + threadIdx.x;
+  const uint64_t step = blockDim.x;
+  for (; i + (U - 1) * step < hi; i += U * step) {
+    uint4 va[U], vb[U];
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      va[u] = ld_stream(a + i + u * step);
+      if (b) vb[u] = ld_stream(b + i + u * step);
+    }
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      x ^= va[u].x ^ va[u].y ^ va[u].z ^ va[u].w;
+      if (b) x ^= vb[u].x ^ vb[u].y ^ vb[u].z ^ vb[u].w;
+    }
+  }
+  for (; i < hi; i += step) {
+    const uint4 va = ld_stream(a + i);
+    x ^= va.x ^ va.y ^ va.z ^ va.w;
+    if (b) {
+      const uint4 vb = ld_stream(b + i);
+      x ^= vb.x ^ vb.y ^ vb.z ^ vb.w;
+    }
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) x ^= __shfl_xor_sync(0xffffffffu, x, o);
+  __shared__ uint32_t s_x[32];
+  if ((threadIdx.x & 31) == 0) s_x[threadIdx.x >> 5] = x;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    uint32_t t = 0;
+    for (int w = 0; w < (int)(blockDim.x >> 5); ++w) t ^= s_x[w];
+    sink[blockIdx.x] = t;
+  }
+}
+
 }  // namespace stride
+
+extern "C" STRIDE_API int stride_selftest_stream_read(const void* a, const void* b, uint64_t bytes_each,
+                                                      int32_t grid, int32_t threads, uint32_t* sink,
+                                                      void* stream) {
+  if (!a || !sink || bytes_each == 0 || (bytes_each & 15u) != 0) return STRIDE_ERR_INVALID_ARG;
+  if ((reinterpret_cast<uintptr_t>(a) & 15u) != 0 || (reinterpret_cast<uintptr_t>(b) & 15u) != 0)
+    return STRIDE_ERR_INVALID_ARG;
+  if (grid < 1 || threads < 32 || threads > 1024 || (threads & 31) != 0) return STRIDE_ERR_INVALID_ARG;
+  if (bytes_each / 16 > UINT64_MAX / (uint64_t)grid) return STRIDE_ERR_INVALID_ARG;  // slice bounds in 64 bits
+  stride::stream_read_kernel<<<(unsigned)grid, (unsigned)threads, 0, (cudaStream_t)stream>>>(
+      reinterpret_cast<const uint4*>(a), reinterpret_cast<const uint4*>(b), bytes_each / 16, sink);
+  return cudaGetLastError() == cudaSuccess ? STRIDE_OK : STRIDE_ERR_CUDA;
+}
 
 extern "C" STRIDE_API int stride_selftest_bounded_wait(int32_t which, uint64_t timeout_ns,
                                                        int32_t* dev_status, void* workspace,

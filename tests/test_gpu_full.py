@@ -7,7 +7,8 @@ configurations the library is used in, against the oracle on every row.
   with the carried state, then the restart choice over its turn statistics
   with Bernoulli(0.5) and Bernoulli(0.9) masks, alpha = -inf and -6.0;
 * multi-teacher (128 x 12 turns, 436,156 rows, two teacher streams): streamed
-  in 16,384-row windows;
+  in 16,384-row windows, with one aligned teacher buffer and with the
+  teacher rows in one buffer per domain (the gather-free entry point);
 * the batch-scoring rows again through the vocabulary-sharded path (the
   bench's 4 shards: partial passes, combine, scan on log-probs), on the same
   resident logits.
@@ -94,10 +95,48 @@ def sharded_scan(stride, S, T, tok, offs, lay, lam, n_shards):
     return g
 
 
-def stream_and_score(stride, w, lam, chunk_rows, resident=False, vocab_shards=0):
+class DomainTeachers:
+    """Each domain's teacher rows in a buffer of their own (trajectories in
+    order), filled window by window from the generated rows: the layout
+    stride_score_batch_multi_teacher reads without a gather."""
+
+    def __init__(self, w, dev):
+        import torch
+
+        lay = w.layout
+        self.dom = w.extra["domain"].astype(np.uint8)
+        n_rows = np.diff(lay.traj_row_off)
+        self.row0 = np.zeros(lay.n_traj, np.int64)
+        self.bufs = []
+        for j in range(2):
+            sel = self.dom == j
+            self.row0[sel] = np.concatenate([[0], np.cumsum(n_rows[sel])[:-1]])
+            self.bufs.append(torch.empty((int(n_rows[sel].sum()), w.recipe.V), dtype=torch.bfloat16, device=dev))
+        self.traj_domain = torch.from_numpy(self.dom).to(dev)
+        self.traj_T_row0 = torch.from_numpy(self.row0).to(dev)
+        self.row_traj = lay.row_traj()
+        self.traj_row_off = lay.traj_row_off
+        self.dev = dev
+
+    def fill(self, T, a, b):
+        """Scatter teacher rows T (window rows [a, b)) to their domain buffers."""
+        import torch
+
+        rt = self.row_traj[a:b]
+        dest = self.row0[rt] + (np.arange(a, b) - self.traj_row_off[rt])
+        for j in range(2):
+            m = np.nonzero(self.dom[rt] == j)[0]
+            if m.size:
+                self.bufs[j].index_copy_(0, torch.from_numpy(dest[m]).to(self.dev),
+                                         T.index_select(0, torch.from_numpy(m).to(self.dev)))
+
+
+def stream_and_score(stride, w, lam, chunk_rows, resident=False, vocab_shards=0, domain_teachers=False):
     """Generate the workload window by window on the GPU, score each window
     with the carried state, and run the oracle on the same rows (and, on a
-    resident workload, the vocabulary-sharded path too)."""
+    resident workload, the vocabulary-sharded path too).  domain_teachers:
+    score through stride_score_batch_multi_teacher, the teacher rows read
+    from one buffer per domain."""
     import torch
 
     lay = w.layout
@@ -119,19 +158,31 @@ def stream_and_score(stride, w, lam, chunk_rows, resident=False, vocab_shards=0)
     tok = torch.empty(win, dtype=torch.int32, device=dev)
     out = {k: torch.empty(win, dtype=torch.float32, device=dev) for k in keys}
     windows = [(0, R)] if resident else [(a, min(R, a + chunk_rows)) for a in range(0, R, chunk_rows)]
+    if domain_teachers:
+        doms = DomainTeachers(w, dev)
+        ws = torch.empty(stride.multi_teacher_workspace_size(win), dtype=torch.uint8, device=dev)
     for a, b in windows:
         n = b - a
         gen = 8192
         for c in range(0, n, gen):
             d = min(n, c + gen)
             synth.generate_rows(w.recipe, a + c, d - c, device=dev, out_S=S[c:d], out_T=T[c:d], out_tok=tok[c:d])
-        stride.stride_score_batch(S[:n], T[:n], tok[:n], *offs, a, b, stride.TURN_MEAN, float(lam), st,
-                                  out={k: v[:n] for k, v in out.items()}, turn_stats=ts, dev_status=status,
-                                  workspace=ws, profile=prof)
+        o_win = {k: v[:n] for k, v in out.items()}
+        if domain_teachers:
+            doms.fill(T[:n], a, b)
+            oracle_rows(copier, S[:n], T[:n], tok[:n], o, a)
+            T[:n].fill_(float("nan"))  # the scoring must not read the aligned copy
+            stride.stride_score_batch_multi_teacher(S[:n], doms.bufs, doms.traj_domain, doms.traj_T_row0, tok[:n],
+                                                    *offs, a, b, stride.TURN_MEAN, float(lam), st, out=o_win,
+                                                    turn_stats=ts, dev_status=status, workspace=ws, profile=prof)
+        else:
+            stride.stride_score_batch(S[:n], T[:n], tok[:n], *offs, a, b, stride.TURN_MEAN, float(lam), st,
+                                      out=o_win, turn_stats=ts, dev_status=status, workspace=ws, profile=prof)
         torch.cuda.synchronize()
         for k in keys:
             g[k][a:b] = out[k][:n].cpu().numpy()
-        oracle_rows(copier, S[:n], T[:n], tok[:n], o, a)
+        if not domain_teachers:
+            oracle_rows(copier, S[:n], T[:n], tok[:n], o, a)
     g["state"] = stride.state_to_numpy(st)[: lay.n_traj]
     g["turn_stats"] = stride.turn_stats_to_numpy(ts)[: lay.n_turns]
     g["status"] = int(status.item())
@@ -202,4 +253,16 @@ def test_full_multi_teacher_chunked(stride):
     w = synth.multi_teacher()
     cal = synth.load_calibration(w.name)
     g, o = stream_and_score(stride, w, cal["lambda"], w.extra["chunk_rows"])
+    _check(g, o, w.layout, cal["lambda"], cal["early_stop_fraction"])
+
+
+def test_full_multi_teacher_domain_buffers(stride):
+    """The multi-teacher workload as Sec. 5.3 scores it: each trajectory
+    against its own domain's teacher, the teacher rows of the two domains in
+    two buffers of their own, through stride_score_batch_multi_teacher (no
+    gather), in the bench's 16,384-row windows; every row, turn and
+    trajectory against the oracle."""
+    w = synth.multi_teacher()
+    cal = synth.load_calibration(w.name)
+    g, o = stream_and_score(stride, w, cal["lambda"], w.extra["chunk_rows"], domain_teachers=True)
     _check(g, o, w.layout, cal["lambda"], cal["early_stop_fraction"])
