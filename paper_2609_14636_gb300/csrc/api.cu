@@ -401,7 +401,11 @@ int stride_scan_logprobs(const float* logp_s, const float* logp_t, const int64_t
   p.incl = reinterpret_cast<stride::ScanSlot*>(ws + L.incl_off);
   p.timeout_ns = 2000000000ull;
   cudaStream_t st = (cudaStream_t)stream;
-  if (cudaMemsetAsync(workspace, 0, L.clear_bytes, st) != cudaSuccess) return STRIDE_ERR_CUDA;
+  int sm_dev = 0;
+  cudaError_t sm_err = cudaSuccess;
+  const int sms = stride::current_device_sms(&sm_dev, &sm_err);
+  if (sms <= 0) return STRIDE_ERR_CUDA;
+  if (stride::launch_clear_workspace(workspace, L.clear_bytes, sms, st) != cudaSuccess) return STRIDE_ERR_CUDA;
   return stride::launch_scan_logprobs(p, logp_s, logp_t, st) == cudaSuccess ? STRIDE_OK : STRIDE_ERR_CUDA;
 }
 

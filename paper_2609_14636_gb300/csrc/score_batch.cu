@@ -135,7 +135,10 @@ template <typename LT, bool VEC>
 __global__ void __launch_bounds__(kSplitThreads, kSplitBlocksPerSm)
     score_batch_split_kernel(const BatchParams p) {
   __shared__ float s_red[4][kSplitWarps];
-  __shared__ float s_part[4];
+  __shared__ float4 s_part[kSplitMaxCluster];  // rank 0: every rank's (mS, sS, mT, sT), written by the ranks
+  // first cluster-barrier phase: waited on before the first remote store
+  // (every CTA of the cluster has started by then)
+  cluster_arrive_relaxed();
   // Launched as a programmatic dependent of the previous kernel on the
   // stream: the CTAs may be scheduled while it finishes, and each waits for
   // its completion before the first global access.  Only then may the
@@ -194,31 +197,31 @@ __global__ void __launch_bounds__(kSplitThreads, kSplitBlocksPerSm)
     s_red[3][warp] = sT;
   }
   __syncthreads();
+  cluster_wait_acquire();  // (first phase) every CTA of the cluster has started
   if (warp == 0) {
     mS = lane < kSplitWarps ? s_red[0][lane] : kMaxStart;
     sS = lane < kSplitWarps ? s_red[1][lane] : 0.f;
     mT = lane < kSplitWarps ? s_red[2][lane] : kMaxStart;
     sT = lane < kSplitWarps ? s_red[3][lane] : 0.f;
     warp_merge2(mS, sS, mT, sT);
-    if (lane == 0) {
-      s_part[0] = mS;
-      s_part[1] = sS;
-      s_part[2] = mT;
-      s_part[3] = sT;
-    }
+    if (lane == 0) cluster.map_shared_rank(s_part, 0)[rank] = make_float4(mS, sS, mT, sT);
   }
-  cluster.sync();
-  if (rank == 0 && warp == 0) {
+  // second phase: the ranks' pairs are released to rank 0; the other ranks
+  // leave (nobody reads their shared memory)
+  cluster_arrive_release();
+  if (rank != 0) return;
+  cluster_wait_acquire();
+  if (warp == 0) {
     mS = kMaxStart;
     sS = 0.f;
     mT = kMaxStart;
     sT = 0.f;
     if (lane < n_ranks) {
-      const float* peer = cluster.map_shared_rank(s_part, lane);
-      mS = peer[0];
-      sS = peer[1];
-      mT = peer[2];
-      sT = peer[3];
+      const float4 q = s_part[lane];
+      mS = q.x;
+      sS = q.y;
+      mT = q.z;
+      sT = q.w;
     }
     warp_merge2(mS, sS, mT, sT);
     if (lane == 0) {
@@ -236,7 +239,6 @@ __global__ void __launch_bounds__(kSplitThreads, kSplitBlocksPerSm)
       p.ws_logp_t[tile] = lpt;
     }
   }
-  cluster.sync();  // the ranks' shared memory has been read: they may leave
 }
 
 // Multi-teacher pre-pass: the teacher row of each window row, from its
@@ -367,6 +369,41 @@ static cudaError_t launch_split(const BatchParams& p, int C, cudaStream_t stream
   return cudaLaunchKernelEx(&cfg, score_batch_split_kernel<LT, VEC>, p);
 }
 
+// Clears what a batch call needs at zero in its workspace (the ticket and
+// the scan flags), launched as a programmatic dependent of the previous
+// kernel on the stream: its CTAs wait for that kernel (which may be the
+// previous window's scoring kernel, still using the same workspace) before
+// the first store.  It lets its own dependent, the scoring kernel, be
+// scheduled at once: that kernel's CTAs set up their shared memory and
+// barriers while the previous window drains, then wait for this grid to
+// complete.  (It replaces a memset node, which ended the programmatic chain:
+// 7.5 us between one 16,384-row window's last CTA and the next one's first
+// on GB300.)
+__global__ void clear_workspace_kernel(uint4* __restrict__ p, int64_t n16) {
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+  const uint4 z = make_uint4(0u, 0u, 0u, 0u);
+  for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n16; i += (int64_t)gridDim.x * blockDim.x)
+    p[i] = z;
+}
+
+cudaError_t launch_clear_workspace(void* ws, size_t bytes, int sms, cudaStream_t stream) {
+  const int64_t n16 = (int64_t)(bytes / 16);  // workspace offsets are 256-byte multiples
+  if (n16 <= 0) return cudaSuccess;
+  int64_t blocks = (n16 + 255) / 256;
+  if (blocks > 2 * (int64_t)sms) blocks = 2 * (int64_t)sms;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)blocks);
+  cfg.blockDim = dim3(256);
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, clear_workspace_kernel, reinterpret_cast<uint4*>(ws), n16);
+}
+
 cudaError_t launch_score_batch(const BatchParams& p, int dtype, bool vec, size_t clear_bytes, cudaStream_t stream) {
   // Small windows split each row over a cluster (split_cluster); 16-byte-
   // aligned rows with at least one whole vector otherwise take the
@@ -402,7 +439,7 @@ cudaError_t launch_score_batch(const BatchParams& p, int dtype, bool vec, size_t
     return launch_scan_logprobs(q, p.ws_logp_s, p.ws_logp_t, stream, true);
   }
   {
-    const cudaError_t e = cudaMemsetAsync(p.ticket, 0, clear_bytes, stream);
+    const cudaError_t e = launch_clear_workspace(p.ticket, clear_bytes, sms, stream);
     if (e != cudaSuccess) return e;
   }
   const int per_vec = dtype == STRIDE_DTYPE_BF16 ? 8 : 4;

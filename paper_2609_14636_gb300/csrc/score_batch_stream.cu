@@ -137,6 +137,12 @@ __global__ void __launch_bounds__(kStreamThreads, 1) score_batch_stream_kernel(c
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
   __syncthreads();
+  // Launched as a programmatic dependent of the workspace clear: the set-up
+  // above may overlap the previous kernel's end; nothing global is touched
+  // before the clear (and everything before it) has completed.  Dependents
+  // may be scheduled at once: they wait for this grid in turn.
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 
   if (warp == 0) {
     // ------------------------------------------------------------ producer
@@ -404,10 +410,19 @@ cudaError_t launch_score_batch_stream(const BatchParams& p, int dtype, cudaStrea
     attr_done[dev][di].store(true, std::memory_order_release);
   }
   const int64_t grid = p.n_rows < sms ? p.n_rows : sms;
-  if (dtype == STRIDE_DTYPE_BF16)
-    score_batch_stream_kernel<__nv_bfloat16><<<(unsigned)grid, kStreamThreads, kStreamSmem, stream>>>(p);
-  else
-    score_batch_stream_kernel<float><<<(unsigned)grid, kStreamThreads, kStreamSmem, stream>>>(p);
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)grid);
+  cfg.blockDim = dim3(kStreamThreads);
+  cfg.dynamicSmemBytes = kStreamSmem;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  e = dtype == STRIDE_DTYPE_BF16 ? cudaLaunchKernelEx(&cfg, score_batch_stream_kernel<__nv_bfloat16>, p)
+                                 : cudaLaunchKernelEx(&cfg, score_batch_stream_kernel<float>, p);
+  if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }
 

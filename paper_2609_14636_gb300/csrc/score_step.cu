@@ -78,18 +78,6 @@ __device__ __forceinline__ void write_row_nan(const StepParams& p, int b) {
 
 }  // namespace
 
-// Cluster barrier halves (PTX barrier.cluster): every thread of the cluster
-// arrives; a wait returns once all non-exited threads have arrived.
-__device__ __forceinline__ void cluster_arrive_relaxed() {
-  asm volatile("barrier.cluster.arrive.relaxed.aligned;" ::: "memory");
-}
-__device__ __forceinline__ void cluster_arrive_release() {
-  asm volatile("barrier.cluster.arrive.release.aligned;" ::: "memory");
-}
-__device__ __forceinline__ void cluster_wait_acquire() {
-  asm volatile("barrier.cluster.wait.acquire.aligned;" ::: "memory");
-}
-
 // The 80-byte state as ten 8-byte L2 loads (no L1: the previous step's
 // cluster wrote it on another SM), issued together.
 __device__ __forceinline__ stride_scan_state load_state(const stride_scan_state* sp) {

@@ -266,6 +266,20 @@ __device__ __forceinline__ uint64_t globaltimer_ns() {
   return t;
 }
 
+// Cluster barrier halves (PTX barrier.cluster, executed by every thread of
+// the CTA): a wait returns once all non-exited threads of the cluster have
+// arrived.  Arriving at kernel start and waiting before the first remote
+// shared-memory store guarantees the target CTA has started.
+__device__ __forceinline__ void cluster_arrive_relaxed() {
+  asm volatile("barrier.cluster.arrive.relaxed.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void cluster_arrive_release() {
+  asm volatile("barrier.cluster.arrive.release.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void cluster_wait_acquire() {
+  asm volatile("barrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+
 __device__ __forceinline__ void set_status(int32_t* dev_status, int bits) {
   if (dev_status) atomicOr(dev_status, bits);
 }

@@ -140,6 +140,9 @@ int current_device_sms(int* dev_out, cudaError_t* err);
 // launches the batch scoring kernels.
 cudaError_t launch_score_batch(const BatchParams& p, int dtype, bool vec, size_t clear_bytes, cudaStream_t stream);
 cudaError_t launch_score_batch_stream(const BatchParams& p, int dtype, cudaStream_t stream);
+// Zeroes `bytes` (a multiple of 16) at ws as a programmatic dependent of the
+// previous kernel on the stream (it waits for that kernel first).
+cudaError_t launch_clear_workspace(void* ws, size_t bytes, int sms, cudaStream_t stream);
 cudaError_t launch_score_step(const StepParams& p, int dtype, bool vec, cudaStream_t stream);
 // Diagnostic overrides of the automatic kernel choices (process-wide; 0 on
 // success, -1 for a value out of range).
