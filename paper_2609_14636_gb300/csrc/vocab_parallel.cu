@@ -161,9 +161,23 @@ __global__ void combine_kernel(const float* __restrict__ parts, int32_t n_shards
 constexpr int kRestartTurn = 1;  // st, sd, sl restart at this row
 constexpr int kRestartSum = 2;   // c restarts (a seeded row)
 
+// A row's element inside a tile.  The running stop sum c is fp64 (the stop
+// rule compares it with lambda); the open-turn sums of log pi_T, d and the
+// loss term are fp32 inside the tile (at most kScanTileRows terms each,
+// summed in a tree: relative error a few 1e-7 of the summed magnitudes) and
+// fp64 again once combined with the tile's prefix.  GB300 runs FP64 at 1/64
+// of the FP32 rate, and the tile scans' fp64 adds were what a small window's
+// scan waited on (a 512-row window in one CTA: 6.6 us for the block scan).
 struct TileElem {
-  double c, st, sd, sl;
+  double c;
+  float st, sd, sl;
   int flags;
+};
+
+// A prefix over tiles (the lookback's result, a row's inclusive and
+// exclusive values): fp64 throughout.
+struct PreElem {
+  double c, st, sd, sl;
 };
 
 __device__ __forceinline__ TileElem tile_combine(const TileElem& a, const TileElem& b) {
@@ -173,6 +187,16 @@ __device__ __forceinline__ TileElem tile_combine(const TileElem& a, const TileEl
   r.sd = (b.flags & kRestartTurn) ? b.sd : a.sd + b.sd;
   r.sl = (b.flags & kRestartTurn) ? b.sl : a.sl + b.sl;
   r.flags = a.flags | b.flags;
+  return r;
+}
+
+// A tile's prefix followed by an in-tile prefix.
+__device__ __forceinline__ PreElem pre_combine(const PreElem& a, const TileElem& b) {
+  PreElem r;
+  r.c = (b.flags & kRestartSum) ? b.c : a.c + b.c;
+  r.st = (b.flags & kRestartTurn) ? (double)b.st : a.st + (double)b.st;
+  r.sd = (b.flags & kRestartTurn) ? (double)b.sd : a.sd + (double)b.sd;
+  r.sl = (b.flags & kRestartTurn) ? (double)b.sl : a.sl + (double)b.sl;
   return r;
 }
 
@@ -190,7 +214,7 @@ __device__ __forceinline__ TileElem tile_shfl_up(const TileElem& v, int d) {
 // retained rows' loss terms and count, and whether a row crossed lambda.
 // Restarts at a trajectory's first row.
 struct TrajElem {
-  double loss;
+  float loss;  // a tile's rows only; added to the fp64 record
   int count;
   int crossed;
   int restart;
@@ -272,7 +296,7 @@ __global__ void __launch_bounds__(TILE) scan_logprobs_tile_kernel(const BatchPar
   __shared__ TileElem s_wpre[kWarps];
   __shared__ TrajElem s_ttot[kWarps];
   __shared__ TrajElem s_tpre[kWarps];
-  __shared__ TileElem s_excl;
+  __shared__ PreElem s_excl;
   __shared__ TileElem s_agg;
   __shared__ int s_flags;  // bit 0: lookback timed out
   __shared__ double s_prof[3 * STRIDE_PROFILE_BINS];
@@ -415,19 +439,19 @@ __global__ void __launch_bounds__(TILE) scan_logprobs_tile_kernel(const BatchPar
       atomicAdd(s_prof + 3 * jb + 2, 1.0);
     }
     if (seeded && !meta.bad) {
-      x = TileElem{cum0 + ec, st0 + est, sd0 + esd, sl0 + esl, kRestartSum | kRestartTurn};
+      x = TileElem{cum0 + ec, (float)(st0 + est), (float)(sd0 + esd), (float)(sl0 + esl), kRestartSum | kRestartTurn};
       c_before = cum0;
       st_before = st0;
     } else if (seeded) {
-      x = TileElem{ec, est, esd, esl, kRestartSum | kRestartTurn};  // NaN: nothing after a bad row is meaningful
+      x = TileElem{ec, (float)est, (float)esd, (float)esl, kRestartSum | kRestartTurn};  // NaN: nothing after a bad row is meaningful
     } else {
-      x = TileElem{ec, est, esd, esl, fturn ? kRestartTurn : 0};
+      x = TileElem{ec, (float)est, (float)esd, (float)esl, fturn ? kRestartTurn : 0};
     }
     if (seeded) x.flags |= 4;  // bit 2: this row's exclusive prefix is the carried state, not the scan
   }
 
   // 3. segmented inclusive scan over the tile
-  const TileElem tile_id = {0.0, 0.0, 0.0, 0.0, 0};
+  const TileElem tile_id = {0.0, 0.f, 0.f, 0.f, 0};
   TileElem tile_incl, tile_excl;
   block_scan<kWarps>(x, tile_id, lane, warp, s_wtot, s_wpre, tile_incl, tile_excl);
 
@@ -445,15 +469,15 @@ __global__ void __launch_bounds__(TILE) scan_logprobs_tile_kernel(const BatchPar
   __syncthreads();
   if (warp == 0) {
     const TileElem agg = s_agg;
-    TileElem pre = {0.0, 0.0, 0.0, 0.0, 0};
+    PreElem pre = {0.0, 0.0, 0.0, 0.0};
     bool timed_out = false;
     // The rows before the tile's first seeded row need the predecessors' sum
     // (a tile whose first row is seeded needs nothing).
     if (!(__shfl_sync(0xffffffffu, x.flags, 0) & kRestartSum)) {
       const ScanElem e = lookback(p, tile, lane, timed_out);
-      pre = TileElem{e.c, e.st, e.sd, e.sl, 0};
+      pre = PreElem{e.c, e.st, e.sd, e.sl};
       if (lane == 0 && !(agg.flags & kRestartSum)) {
-        const TileElem inc = tile_combine(pre, agg);
+        const PreElem inc = pre_combine(pre, agg);
         ScanElem ie{inc.c, inc.st, inc.sd, inc.sl, 1};
         publish(p.incl + tile, p.flags + tile * kFlagStride, ie, kStIncl);
       }
@@ -467,10 +491,10 @@ __global__ void __launch_bounds__(TILE) scan_logprobs_tile_kernel(const BatchPar
 
   // 5. complete every row
   if (live) {
-    const TileElem pre = s_excl;
-    const TileElem ri = tile_combine(pre, tile_incl);
+    const PreElem pre = s_excl;
+    const PreElem ri = pre_combine(pre, tile_incl);
     if (!(x.flags & 4)) {
-      const TileElem re = tile_combine(pre, tile_excl);
+      const PreElem re = pre_combine(pre, tile_excl);
       c_before = re.c;
       st_before = fturn ? 0.0 : re.st;
     }
@@ -486,7 +510,7 @@ __global__ void __launch_bounds__(TILE) scan_logprobs_tile_kernel(const BatchPar
   //    the stop (the running sum never rises, so it is the trajectory's
   //    first crossing unless an earlier tile's is lower), and the last row
   //    of a trajectory here adds its retained rows' loss and count.
-  TrajElem te = {0.0, 0, 0, 1};
+  TrajElem te = {0.f, 0, 0, 1};
   bool cross = false;
   if (live && !meta.bad) {
     const int64_t n_k = meta.turn_end - meta.turn_start;
@@ -495,9 +519,9 @@ __global__ void __launch_bounds__(TILE) scan_logprobs_tile_kernel(const BatchPar
     cross = test && ri_c < (double)lam;
     const double before = (p.mode == STRIDE_STOP_TOKEN_SUM) ? c_before : c_before - st_before / (double)n_k;
     const bool kept = before >= (double)lam;
-    te = TrajElem{kept ? e_sl : 0.0, kept ? 1 : 0, cross ? 1 : 0, r == meta.traj_start ? 1 : 0};
+    te = TrajElem{kept ? (float)e_sl : 0.f, kept ? 1 : 0, cross ? 1 : 0, r == meta.traj_start ? 1 : 0};
   }
-  const TrajElem traj_id = {0.0, 0, 0, 0};
+  const TrajElem traj_id = {0.f, 0, 0, 0};
   TrajElem t_incl, t_excl;
   block_scan<kWarps>(te, traj_id, lane, warp, s_ttot, s_tpre, t_incl, t_excl);
   if (live && !meta.bad) {
