@@ -363,11 +363,18 @@ __global__ void __launch_bounds__(kStreamThreads, 1) score_batch_stream_kernel(c
   for (int64_t seq = warp - 2;; seq += kScanWarps) {
     const int q = (int)(seq % kSlots);
     const uint32_t use = (uint32_t)(seq / kSlots);
-    // wait for row `seq`, unless the rows ran out before it
-    bool ready = mbar_try_wait(&sh.agg_ready[q], use & 1u);
+    // Wait for row `seq`, unless the rows ran out before it.  The slots
+    // past the last row never fill, so the wait polls (test_wait and a short
+    // sleep) and looks at the end marker in between: a blocking try_wait
+    // kept each scan warp suspended about 7.5 us after the row warp had
+    // marked the end (probe timeline of 16,384-row windows: every CTA left
+    // 7.4-7.7 us after its scan warps began their last wait).
+    if (*end_seq <= seq) break;
+    bool ready = mbar_test_wait(&sh.agg_ready[q], use & 1u);
     if (!ready) {
       const uint64_t t0 = globaltimer_ns();
-      while (!(ready = mbar_try_wait(&sh.agg_ready[q], use & 1u))) {
+      while (!(ready = mbar_test_wait(&sh.agg_ready[q], use & 1u))) {
+        __nanosleep(100);
         if (*end_seq <= seq || *abort) break;
         if (globaltimer_ns() - t0 > tmo) {
           if (lane == 0) raise_abort(sh, p);
