@@ -1,0 +1,146 @@
+"""Randomised GPU parity of the batch path: seeded random ragged layouts
+(one-row turns and trajectories included), vocabulary sizes, logit dtypes,
+row strides (aligned or not), stop modes, per-trajectory thresholds placed
+between the oracle's running sums, and row windows cut at random places,
+through the automatic kernel choice and each forced batch kernel; every row,
+turn and trajectory against the oracle under the tolerances of
+gpu_helpers.  And the scan alone (stride_scan_logprobs) on random layouts of
+thousands of rows -- many 256-row tiles, lookbacks across them, seeded rows
+inside tiles -- fed the same fp32 log-probs as the oracle's scan."""
+from __future__ import annotations
+
+import numpy as np
+import pytest
+
+import synth
+from gpu_helpers import compare_rows, compare_scan, oracle_batch, pad_cols, run_batch
+
+pytestmark = pytest.mark.gpu
+
+SEEDS = list(range(40))
+VOCABS = (257, 1000, 4099, 8192, 32_000)
+
+
+@pytest.fixture(scope="module")
+def stride():
+    import paper_2609_14636_gb300 as s
+
+    return s
+
+
+def _case(seed):
+    rng = np.random.default_rng(1000 + seed)
+    n_traj = int(rng.integers(1, 7))
+    lens = []
+    for _ in range(n_traj):
+        nt = int(rng.integers(1, 6))
+        lens.append([1 if rng.random() < 0.25 else int(rng.integers(2, 121)) for _ in range(nt)])
+    lay = synth.layout_from_turn_lengths(lens)
+    R = lay.rows
+    V = int(rng.choice(VOCABS))
+    while R * V > 12_000_000 and V > VOCABS[0]:
+        V = max(v for v in VOCABS if v < V)
+    f32 = bool(rng.random() < 0.4)
+    ld = V + (int(rng.integers(1, 10)) if rng.random() < 0.4 else 0)
+    mode = int(rng.integers(0, 2))
+    sigma = float(rng.uniform(1.0, 5.0))
+    S32 = rng.standard_normal((R, V), dtype=np.float32) * np.float32(sigma)
+    T32 = S32 + rng.standard_normal((R, V), dtype=np.float32) * np.float32(rng.uniform(0.2, 2.0))
+    if f32:
+        S, T = S32, T32.astype(np.float32)
+        fill = np.float32(np.nan)
+    else:
+        S = synth.bf16_bits_from_f32(S32)
+        T = synth.bf16_bits_from_f32(synth.f32_from_bf16_bits(S) + (T32 - S32))
+        fill = 0x7FC0  # NaN padding: never read
+    tok = rng.integers(0, V, R).astype(np.int32)
+    n_cuts = int(rng.integers(0, 4))
+    cuts = sorted(set([0, R] + [int(x) for x in rng.integers(1, R, size=n_cuts)] if R > 1 else [0, R]))
+    windows = list(zip(cuts[:-1], cuts[1:]))
+    return lay, S, T, tok, V, ld, mode, windows, fill, rng
+
+
+def _lambda(o, lay, mode, rng):
+    """Per-trajectory thresholds halfway between two of the oracle's
+    consecutive test values (or below all of them), so that about half the
+    trajectories stop, none inside the tie band."""
+    lam = np.empty(lay.n_traj, np.float32)
+    for i in range(lay.n_traj):
+        if mode == 1:
+            r0, r1 = lay.traj_row_off[i], lay.traj_row_off[i + 1]
+            vals = o["row_cum"][r0:r1]
+        else:
+            vals = o["turn_cum"][lay.traj_turn_off[i]:lay.traj_turn_off[i + 1]]
+        if rng.random() < 0.5 or len(vals) == 1:
+            lam[i] = np.float32(vals[-1] - 1.0)  # never crosses
+        else:
+            t = int(rng.integers(1, len(vals)))
+            lam[i] = np.float32(0.5 * (vals[t - 1] + vals[t]))
+    return lam
+
+
+@pytest.mark.parametrize("kernel", ["auto", "stream", "split", "rows"])
+@pytest.mark.parametrize("seed", SEEDS)
+def test_random_layouts(stride, seed, kernel):
+    lay, S, T, tok, V, ld, mode, windows, fill, rng = _case(seed)
+    o0 = oracle_batch(S, T, tok, lay, mode, np.float32(-1e30))
+    lam = _lambda(o0, lay, mode, rng)
+    o = oracle_batch(S, T, tok, lay, mode, lam)
+    Sp, Tp = (S, T) if ld == V else (pad_cols(S, ld, fill), pad_cols(T, ld, fill))
+    stride.stride_force_batch_kernel(kernel)
+    try:
+        g = run_batch(stride, Sp, Tp, tok, lay, mode, lam, windows=windows, V=V)
+    finally:
+        stride.stride_force_batch_kernel("auto")
+    assert g["status"] == 0
+    compare_rows(g, o)
+    compare_scan(g, o, lay, mode, lam)
+
+
+@pytest.mark.parametrize("seed", list(range(12)))
+def test_random_scan_on_logprobs(stride, seed):
+    import torch
+
+    import oracle
+
+    rng = np.random.default_rng(5000 + seed)
+    n_traj = int(rng.integers(1, 40))
+    lens = []
+    for _ in range(n_traj):
+        nt = int(rng.integers(1, 12))
+        lens.append([1 if rng.random() < 0.2 else int(rng.integers(2, 700)) for _ in range(nt)])
+    lay = synth.layout_from_turn_lengths(lens)
+    R = lay.rows
+    mode = int(rng.integers(0, 2))
+    # log-probs as the scan receives them (fp32, <= 0)
+    lpt = (-np.abs(rng.standard_normal(R)) * rng.uniform(1.0, 8.0)).astype(np.float32)
+    lps = (lpt + rng.standard_normal(R).astype(np.float32) * np.float32(0.7)).astype(np.float32)
+    lps = np.minimum(lps, np.float32(0.0))
+    d = (lps.astype(np.float64) - lpt.astype(np.float64))
+    o0 = oracle.scan_batch(lpt.astype(np.float64), d, lay.traj_row_off, lay.turn_row_off, lay.traj_turn_off,
+                           mode, np.float64(-1e30), logp_s=lps.astype(np.float64))
+    o0.update(logp_t=lpt.astype(np.float64), d=d)
+    lam = _lambda(o0, lay, mode, rng)
+    o = oracle.scan_batch(lpt.astype(np.float64), d, lay.traj_row_off, lay.turn_row_off, lay.traj_turn_off,
+                          mode, lam.astype(np.float64), logp_s=lps.astype(np.float64))
+    o.update(logp_t=lpt.astype(np.float64), logp_s=lps.astype(np.float64), d=d)
+    dev = "cuda"
+    offs = [torch.from_numpy(a).to(dev) for a in (lay.traj_row_off, lay.turn_row_off, lay.traj_turn_off)]
+    st = stride.new_state(lay.n_traj)
+    ts = stride.new_turn_stats(lay.n_turns)
+    prof = stride.new_profile(dev)
+    opd = torch.empty(R, dtype=torch.float32, device=dev)
+    status = torch.zeros(1, dtype=torch.int32, device=dev)
+    n_cuts = int(rng.integers(0, 4))
+    cuts = sorted(set([0, R] + [int(x) for x in rng.integers(1, R, size=n_cuts)]))
+    ws = torch.empty(stride.stride_score_batch_workspace_size(R), dtype=torch.uint8, device=dev)
+    lps_d, lpt_d = torch.from_numpy(lps).to(dev), torch.from_numpy(lpt).to(dev)
+    for a, b in zip(cuts[:-1], cuts[1:]):
+        stride.stride_scan_logprobs(lps_d[a:b], lpt_d[a:b], *offs, a, b, mode, torch.from_numpy(lam).to(dev), st,
+                                    opd=opd[a:b], turn_stats=ts, dev_status=status, workspace=ws, profile=prof)
+    torch.cuda.synchronize()
+    g = {"opd": opd.cpu().numpy(), "state": stride.state_to_numpy(st)[: lay.n_traj],
+         "turn_stats": stride.turn_stats_to_numpy(ts)[: lay.n_turns], "profile": prof.cpu().numpy()}
+    assert int(status.item()) == 0
+    assert np.max(np.abs(g["opd"] - d)) <= 2e-3
+    compare_scan(g, o, lay, mode, lam)
