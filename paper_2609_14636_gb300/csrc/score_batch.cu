@@ -248,6 +248,12 @@ __global__ void __launch_bounds__(kSplitThreads, kSplitBlocksPerSm)
 __global__ void teacher_rows_kernel(const BatchParams p, const TeacherTable tt,
                                     const uint8_t* __restrict__ traj_domain,
                                     const int64_t* __restrict__ traj_T_row0, const void** rows_out) {
+  // A programmatic dependent of the previous kernel, which may be the
+  // previous window's scoring kernel still reading this workspace's table:
+  // wait for it before the first store; the clearing and scoring kernels
+  // that follow may be scheduled at once (they wait for this grid in turn).
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
   const int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
   if (t >= p.n_rows) return;
   const int64_t r = p.row_begin + t;
@@ -269,8 +275,17 @@ __global__ void teacher_rows_kernel(const BatchParams p, const TeacherTable tt,
 
 cudaError_t launch_teacher_rows(const BatchParams& p, const TeacherTable& tt, const uint8_t* traj_domain,
                                 const int64_t* traj_T_row0, const void** rows_out, cudaStream_t stream) {
-  const unsigned grid = (unsigned)((p.n_rows + 255) / 256);
-  teacher_rows_kernel<<<grid, 256, 0, stream>>>(p, tt, traj_domain, traj_T_row0, rows_out);
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)((p.n_rows + 255) / 256));
+  cfg.blockDim = dim3(256);
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  const cudaError_t e = cudaLaunchKernelEx(&cfg, teacher_rows_kernel, p, tt, traj_domain, traj_T_row0, rows_out);
+  if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }
 
