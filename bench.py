@@ -401,7 +401,14 @@ class BatchRun:
             ev[1].record(stream)
 
     def launches_per_step(self) -> int:
-        return 1 + len(self.windows) * (1 if self.entry == "aligned" else 2)
+        """The library's kernels in one step: the state init, then per window
+        either the workspace clear and the persistent kernel (windows above
+        8 rows per SM) or the small-window kernel and its scan, plus the
+        teacher-row pre-pass on the multi-teacher path."""
+        per = 2 * len(self.windows)  # clear + persistent, or split + scan
+        if self.entry != "aligned":
+            per += len(self.windows)
+        return 1 + per
 
     def early_fraction(self) -> float:
         st = self.stride.state_to_numpy(self.st)[: self.lay.n_traj]
