@@ -304,3 +304,58 @@ def test_step_full_decode_workload(stride, form):
         r = run_steps(stride, S, T, tok, w["turn_end"], ring, B, mode, lam, V, o_rows, form=form)
         assert r["stopped"] > 0
         assert r["rows"] < B * w["turn_end"].shape[0]
+
+
+@pytest.mark.parametrize("threads,C", [(128, 4), (128, 12), (512, 8)])
+def test_compact_equals_masked_bitwise(stride, threads, C):
+    """With the launch shape fixed, the compacted form computes each live
+    row exactly as the masked form does (same slices, same merge order, same
+    state arithmetic): outputs and carried state bit-identical over a run in
+    which rollouts stop."""
+    import torch
+
+    ring, B, steps, V = 3, 48, 120, 8192
+    S, T, tok, Sp, Tp = _ring(31 + C, ring, B, V, V)
+    rng = np.random.default_rng(C)
+    turn_end = (rng.random((steps, B)) < 1 / 10).astype(np.uint8)
+    St, Tt = to_dev(Sp), to_dev(Tp)
+    tk = torch.from_numpy(tok).cuda()
+    st_m, st_c = stride.new_state(B), stride.new_state(B)
+    keys = ("logp_s", "logp_t", "opd", "lse_s", "lse_t")
+    om = {k: torch.empty(B, dtype=torch.float32, device="cuda") for k in keys}
+    oc = {k: torch.empty(B, dtype=torch.float32, device="cuda") for k in keys}
+    sn_m = torch.empty(B, dtype=torch.uint8, device="cuda")
+    sn_c = torch.empty(B, dtype=torch.uint8, device="cuda")
+    tm = torch.empty((B, stride.TURN_STATS_DTYPE.itemsize), dtype=torch.uint8, device="cuda")
+    tc = torch.empty((B, stride.TURN_STATS_DTYPE.itemsize), dtype=torch.uint8, device="cuda")
+    stopped = np.zeros(B, bool)
+    n_stops = 0
+    stride.stride_force_step_shape(threads, C)
+    try:
+        for s in range(steps):
+            j = s % ring
+            Sj, Tj, kj = St[j * B:(j + 1) * B], Tt[j * B:(j + 1) * B], tk[j * B:(j + 1) * B]
+            te = torch.from_numpy(np.ascontiguousarray(turn_end[s])).cuda()
+            stride.stride_score_step(Sj, Tj, kj, te, 0, -25.0, st_m, out=om, stopped_now=sn_m, turn_out=tm)
+            idx = np.nonzero(~stopped)[0].astype(np.int32)
+            n = idx.shape[0]
+            if n == 0:
+                break
+            it = torch.from_numpy(idx).cuda()
+            stride.stride_score_step_compact(Sj.index_select(0, it), Tj.index_select(0, it), kj.index_select(0, it),
+                                             te.index_select(0, it.long()), it, 0, -25.0, st_c, out=oc,
+                                             stopped_now=sn_c, turn_out=tc)
+            torch.cuda.synchronize()
+            for k in keys:
+                a = om[k].cpu().numpy()[idx].view(np.uint32)
+                b = oc[k][:n].cpu().numpy().view(np.uint32)
+                assert np.array_equal(a, b), (s, k)
+            assert np.array_equal(sn_m.cpu().numpy()[idx], sn_c[:n].cpu().numpy()), s
+            assert np.array_equal(tm.cpu().numpy()[idx], tc[:n].cpu().numpy()), s
+            fired = sn_m.cpu().numpy().astype(bool)
+            n_stops += int(fired.sum())
+            stopped |= fired
+    finally:
+        stride.stride_force_step_shape(0, 0)
+    assert np.array_equal(stride.state_to_numpy(st_m).view(np.uint8), stride.state_to_numpy(st_c).view(np.uint8))
+    assert n_stops > 0
