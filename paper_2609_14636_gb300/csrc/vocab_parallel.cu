@@ -10,8 +10,14 @@
 // log-probs as the full row.  The rest of the path (turn statistics, stop
 // rule, OPD loss, profile, carried state) then runs on the log-probs
 // (scan_logprobs_tile_kernel): a segmented scan per tile of 256 rows, and
-// the fused kernels' decoupled lookback (row_scan.cuh) between tiles.
+// the fused kernels' decoupled lookback (row_scan.cuh) between tiles -- or,
+// for a small window after the small-window kernel, tiles of 128 rows in
+// one thread-block cluster that exchange their aggregates through
+// distributed shared memory.
+#include <cooperative_groups.h>
 #include <math.h>
+
+#include <atomic>
 
 #include "row_scan.cuh"
 #include "stride.h"
@@ -150,7 +156,9 @@ __global__ void combine_kernel(const float* __restrict__ parts, int32_t n_shards
 //   4. the tile's aggregate is published (as an INCLUSIVE prefix at once if
 //      the tile holds a seeded row, since nothing before it matters then;
 //      tile 0 always does), warp 0 folds its predecessors' (row_scan.cuh
-//      lookback) and publishes the tile's inclusive prefix;
+//      lookback) and publishes the tile's inclusive prefix (the cluster
+//      form, below: the aggregates go to the later tiles' shared memory,
+//      and warp 0 folds its predecessors' there);
 //   5. every row completes with its inclusive and exclusive prefixes: turn
 //      statistics and carried state (row_tail), the within-turn profile into
 //      the CTA's shared bins;
@@ -281,7 +289,46 @@ __device__ __forceinline__ int smem_upper_le(const int64_t* a, int n, int64_t r)
   return lo;
 }
 
-template <int TILE>
+// A prefix over tiles with its restart marks (the cluster form's fold of
+// the tiles' aggregates).
+struct PreFlag {
+  double c, st, sd, sl;
+  int flags;
+};
+
+__device__ __forceinline__ PreFlag pre_flag_combine(const PreFlag& a, const PreFlag& b) {
+  PreFlag r;
+  r.c = (b.flags & kRestartSum) ? b.c : a.c + b.c;
+  r.st = (b.flags & kRestartTurn) ? b.st : a.st + b.st;
+  r.sd = (b.flags & kRestartTurn) ? b.sd : a.sd + b.sd;
+  r.sl = (b.flags & kRestartTurn) ? b.sl : a.sl + b.sl;
+  r.flags = a.flags | b.flags;
+  return r;
+}
+
+__device__ __forceinline__ PreFlag pre_flag_shfl(const PreFlag& v, int src) {
+  PreFlag o;
+  o.c = __shfl_sync(0xffffffffu, v.c, src);
+  o.st = __shfl_sync(0xffffffffu, v.st, src);
+  o.sd = __shfl_sync(0xffffffffu, v.sd, src);
+  o.sl = __shfl_sync(0xffffffffu, v.sl, src);
+  o.flags = __shfl_sync(0xffffffffu, v.flags, src);
+  return o;
+}
+
+// The cluster form (CLUSTER; a small window of at most kClusterMaxTiles
+// tiles, launched as ONE thread-block cluster of one CTA per tile, so that
+// the tiles run at once): in place of the lookback through global memory,
+// each tile stores its aggregate into the shared memory of every later
+// tile of the cluster, and after one cluster barrier folds its
+// predecessors' aggregates itself.  A second role of the barrier: the
+// carried state is read before the dependency wait and written at a
+// trajectory's last row, possibly by a later tile, so every CTA arrives
+// once its reads are done and waits before any write.  (In the lookback
+// form that order comes from the chain of published prefixes.)
+constexpr int kClusterMaxTiles = 16;
+
+template <int TILE, bool CLUSTER>
 __global__ void __launch_bounds__(TILE) scan_logprobs_tile_kernel(const BatchParams p,
                                                                           const float* __restrict__ logp_s,
                                                                           const float* __restrict__ logp_t,
@@ -356,6 +403,8 @@ __global__ void __launch_bounds__(TILE) scan_logprobs_tile_kernel(const BatchPar
   }
   __syncthreads();
 
+  __shared__ TileElem s_caggs[CLUSTER ? kClusterMaxTiles : 1];  // (CLUSTER) predecessors' aggregates
+
   // 2. this thread's row: its turn and trajectory, and its element
   RowMeta meta;
   meta.bad = true;
@@ -407,6 +456,7 @@ __global__ void __launch_bounds__(TILE) scan_logprobs_tile_kernel(const BatchPar
     sl0 = fturn ? 0.0 : __ldcg(&sp->turn_sum_l);
   }
   const float lam = (live && !meta.bad) ? (p.lambda ? __ldg(p.lambda + meta.traj) : p.lambda_all) : 0.f;
+  if (CLUSTER) cluster_arrive_release();  // this CTA's reads of the carried state are done
   if (!by_ticket) {
     asm volatile("griddepcontrol.wait;" ::: "memory");
     if (live) {
@@ -414,7 +464,6 @@ __global__ void __launch_bounds__(TILE) scan_logprobs_tile_kernel(const BatchPar
       lpt = __ldcg(logp_t + w);
     }
   }
-
   TileElem x = {0.0, 0.0, 0.0, 0.0, 0};
   double c_before = 0.0, st_before = 0.0, e_sl = 0.0, ri_c = 0.0;
   if (live) {
@@ -455,39 +504,72 @@ __global__ void __launch_bounds__(TILE) scan_logprobs_tile_kernel(const BatchPar
   TileElem tile_incl, tile_excl;
   block_scan<kWarps>(x, tile_id, lane, warp, s_wtot, s_wpre, tile_incl, tile_excl);
 
-  // 4. publish the tile's aggregate, fold predecessors, publish its prefix
-  if (tid == (int)(n_here - 1)) {
-    ScanElem agg{tile_incl.c, tile_incl.st, tile_incl.sd, tile_incl.sl, tile_incl.flags & kRestartTurn};
-    if (tile_incl.flags & kRestartSum) {
-      publish(p.incl + tile, p.flags + tile * kFlagStride, agg, kStIncl);
-    } else {
-      publish(p.agg + tile, p.flags + tile * kFlagStride, agg,
-              kStAgg | ((tile_incl.flags & kRestartTurn) ? kFlagTurnStart : 0u));
+  // 4. the tile's exclusive prefix: from the cluster's other tiles (CLUSTER),
+  //    else publish the tile's aggregate, fold predecessors, publish its prefix
+  if (CLUSTER) {
+    namespace cg = cooperative_groups;
+    if (tid == (int)(n_here - 1)) s_agg = tile_incl;
+    __syncthreads();
+    cluster_wait_acquire();  // every tile has started and read its carried state
+    if (warp == 0) {
+      const cg::cluster_group cl = cg::this_cluster();
+      const TileElem agg = s_agg;
+      for (int64_t j = tile + 1 + lane; j < n_tiles; j += 32) cl.map_shared_rank(s_caggs, (unsigned)j)[tile] = agg;
     }
-    s_agg = tile_incl;  // the aggregate, for warp 0 below
-  }
-  __syncthreads();
-  if (warp == 0) {
-    const TileElem agg = s_agg;
-    PreElem pre = {0.0, 0.0, 0.0, 0.0};
-    bool timed_out = false;
-    // The rows before the tile's first seeded row need the predecessors' sum
-    // (a tile whose first row is seeded needs nothing).
-    if (!(__shfl_sync(0xffffffffu, x.flags, 0) & kRestartSum)) {
-      const ScanElem e = lookback(p, tile, lane, timed_out);
-      pre = PreElem{e.c, e.st, e.sd, e.sl};
-      if (lane == 0 && !(agg.flags & kRestartSum)) {
-        const PreElem inc = pre_combine(pre, agg);
-        ScanElem ie{inc.c, inc.st, inc.sd, inc.sl, 1};
-        publish(p.incl + tile, p.flags + tile * kFlagStride, ie, kStIncl);
+    cluster_arrive_release();
+    cluster_wait_acquire();  // every aggregate has arrived; nothing touches this CTA's memory after
+    if (warp == 0) {
+      PreFlag v = {0.0, 0.0, 0.0, 0.0, 0};
+      if (lane < tile) {
+        const TileElem a = s_caggs[lane];
+        v = PreFlag{a.c, (double)a.st, (double)a.sd, (double)a.sl, a.flags};
+      }
+#pragma unroll
+      for (int d = 1; d < kClusterMaxTiles; d <<= 1) {
+        const PreFlag o = pre_flag_shfl(v, lane >= d ? lane - d : lane);
+        if (lane >= d) v = pre_flag_combine(o, v);
+      }
+      const PreFlag pf = pre_flag_shfl(v, tile > 0 ? (int)tile - 1 : 0);
+      if (lane == 0) {
+        s_excl = tile > 0 ? PreElem{pf.c, pf.st, pf.sd, pf.sl} : PreElem{0.0, 0.0, 0.0, 0.0};
+        s_flags = 0;
       }
     }
-    if (lane == 0) {
-      s_excl = pre;
-      s_flags = timed_out ? 1 : 0;
+    __syncthreads();
+  } else {
+    if (tid == (int)(n_here - 1)) {
+      ScanElem agg{tile_incl.c, tile_incl.st, tile_incl.sd, tile_incl.sl, tile_incl.flags & kRestartTurn};
+      if (tile_incl.flags & kRestartSum) {
+        publish(p.incl + tile, p.flags + tile * kFlagStride, agg, kStIncl);
+      } else {
+        publish(p.agg + tile, p.flags + tile * kFlagStride, agg,
+                kStAgg | ((tile_incl.flags & kRestartTurn) ? kFlagTurnStart : 0u));
+      }
+      s_agg = tile_incl;  // the aggregate, for warp 0 below
     }
+    __syncthreads();
+    if (warp == 0) {
+      const TileElem agg = s_agg;
+      PreElem pre = {0.0, 0.0, 0.0, 0.0};
+      bool timed_out = false;
+      // The rows before the tile's first seeded row need the predecessors' sum
+      // (a tile whose first row is seeded needs nothing).
+      if (!(__shfl_sync(0xffffffffu, x.flags, 0) & kRestartSum)) {
+        const ScanElem e = lookback(p, tile, lane, timed_out);
+        pre = PreElem{e.c, e.st, e.sd, e.sl};
+        if (lane == 0 && !(agg.flags & kRestartSum)) {
+          const PreElem inc = pre_combine(pre, agg);
+          ScanElem ie{inc.c, inc.st, inc.sd, inc.sl, 1};
+          publish(p.incl + tile, p.flags + tile * kFlagStride, ie, kStIncl);
+        }
+      }
+      if (lane == 0) {
+        s_excl = pre;
+        s_flags = timed_out ? 1 : 0;
+      }
+    }
+    __syncthreads();
   }
-  __syncthreads();
 
   // 5. complete every row
   if (live) {
@@ -588,6 +670,38 @@ cudaError_t launch_combine_partials(const float* parts, int32_t n_shards, int64_
   return cudaGetLastError();
 }
 
+// Whether one cluster of n CTAs of the cluster form can be placed on this
+// device (looked up once per device and size; sizes above 8 need the
+// non-portable cluster attribute, set here first).
+bool scan_cluster_fits(int dev, int n, cudaStream_t stream) {
+  constexpr int kMaxDev = 64;
+  static std::atomic<int> fits[kMaxDev][kClusterMaxTiles + 1];  // 0 unknown, 1 yes, 2 no
+  if (dev < 0 || dev >= kMaxDev || n < 1 || n > kClusterMaxTiles) return false;
+  const int known = fits[dev][n].load(std::memory_order_acquire);
+  if (known) return known == 1;
+  auto kern = scan_logprobs_tile_kernel<kScanTileRowsDependent, true>;
+  bool ok = true;
+  if (n > 8) ok = cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) == cudaSuccess;
+  if (ok) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)n);
+    cfg.blockDim = dim3(kScanTileRowsDependent);
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = (unsigned)n;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    int clusters = 0;
+    ok = cudaOccupancyMaxActiveClusters(&clusters, kern, &cfg) == cudaSuccess && clusters >= 1;
+  }
+  if (!ok) (void)cudaGetLastError();  // a refused size is an answer, not an error to carry
+  fits[dev][n].store(ok ? 1 : 2, std::memory_order_release);
+  return ok;
+}
+
 cudaError_t launch_scan_logprobs(const BatchParams& p, const float* logp_s, const float* logp_t,
                                  cudaStream_t stream, bool dependent) {
   // (the small-window path's split kernel cleared the flags of its tiles)
@@ -598,7 +712,7 @@ cudaError_t launch_scan_logprobs(const BatchParams& p, const float* logp_s, cons
   cfg.blockDim = dim3((unsigned)tile_rows);
   cfg.dynamicSmemBytes = 0;
   cfg.stream = stream;
-  cudaLaunchAttribute attr[1];
+  cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
@@ -613,11 +727,23 @@ cudaError_t launch_scan_logprobs(const BatchParams& p, const float* logp_s, cons
   const int sms = current_device_sms(&dev, &qe);
   if (sms <= 0) return qe != cudaSuccess ? qe : cudaErrorInvalidDevice;
   const bool by_ticket = !dependent || n_tiles > sms;
+  // a small dependent window runs as one cluster (the cluster form)
+  const bool cluster = dependent && !by_ticket && n_tiles <= kClusterMaxTiles &&
+                       scan_cluster_fits(dev, (int)n_tiles, stream);
+  if (cluster) {
+    attr[1].id = cudaLaunchAttributeClusterDimension;
+    attr[1].val.clusterDim.x = (unsigned)n_tiles;
+    attr[1].val.clusterDim.y = 1;
+    attr[1].val.clusterDim.z = 1;
+    cfg.numAttrs = 2;
+  }
   const cudaError_t e =
-      dependent ? cudaLaunchKernelEx(&cfg, scan_logprobs_tile_kernel<kScanTileRowsDependent>, p, logp_s, logp_t,
-                                     n_tiles, validate, by_ticket)
-                : cudaLaunchKernelEx(&cfg, scan_logprobs_tile_kernel<kScanTileRows>, p, logp_s, logp_t, n_tiles,
-                                     validate, by_ticket);
+      !dependent ? cudaLaunchKernelEx(&cfg, scan_logprobs_tile_kernel<kScanTileRows, false>, p, logp_s, logp_t,
+                                      n_tiles, validate, by_ticket)
+      : cluster  ? cudaLaunchKernelEx(&cfg, scan_logprobs_tile_kernel<kScanTileRowsDependent, true>, p, logp_s,
+                                      logp_t, n_tiles, validate, by_ticket)
+                 : cudaLaunchKernelEx(&cfg, scan_logprobs_tile_kernel<kScanTileRowsDependent, false>, p, logp_s,
+                                      logp_t, n_tiles, validate, by_ticket);
   if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }

@@ -144,3 +144,53 @@ def test_random_scan_on_logprobs(stride, seed):
     assert int(status.item()) == 0
     assert np.max(np.abs(g["opd"] - d)) <= 2e-3
     compare_scan(g, o, lay, mode, lam)
+
+
+def _window_layout(rng, total, first):
+    """Turn lengths summing to `total` rows: a first trajectory of about
+    `first` rows (several turns), then trajectories of 1-5 turns of 1-200
+    rows (one-row turns among them)."""
+    lens, used = [], 0
+    while used < total:
+        goal = first if not lens else int(rng.integers(1, 600))
+        traj, n = [], 0
+        while n < goal and used + n < total and len(traj) < (40 if not lens else 5):
+            t = 1 if rng.random() < 0.2 else int(rng.integers(2, 201))
+            t = min(t, goal - n, total - used - n)
+            traj.append(max(t, 1))
+            n += traj[-1]
+        lens.append(traj)
+        used += n
+    return synth.layout_from_turn_lengths(lens)
+
+
+@pytest.mark.parametrize("mode", [0, 1])
+@pytest.mark.parametrize("rows", [1, 128, 129, 1024, 1025, 1152, 2047, 2048, 2049])
+def test_small_window_scan_every_cluster_size(stride, rows, mode):
+    """The scan after the small-window kernel at each size class of its
+    launch: windows of 1-16 tiles of 128 rows (one cluster, sizes above 8
+    non-portable) and of 17 tiles (the lookback form); a first trajectory
+    that runs through the whole first window into the second (its state
+    carried into the second window's first tiles, every tile folding all
+    its predecessors' aggregates), short trajectories and one-row turns
+    after it; two windows of `rows` rows, every row, turn and trajectory
+    against the oracle."""
+    rng = np.random.default_rng(9000 + 2 * rows + mode)
+    lay = _window_layout(rng, 2 * rows, first=max(1, (13 * rows) // 10))
+    R = lay.rows
+    assert R == 2 * rows
+    V = 257
+    S = rng.standard_normal((R, V), dtype=np.float32) * np.float32(3.0)
+    T = S + rng.standard_normal((R, V), dtype=np.float32)
+    tok = rng.integers(0, V, R).astype(np.int32)
+    o0 = oracle_batch(S, T, tok, lay, mode, np.float32(-1e30))
+    lam = _lambda(o0, lay, mode, rng)
+    o = oracle_batch(S, T, tok, lay, mode, lam)
+    stride.stride_force_batch_kernel("split")
+    try:
+        g = run_batch(stride, S, T, tok, lay, mode, lam, windows=[(0, rows), (rows, R)], V=V)
+    finally:
+        stride.stride_force_batch_kernel("auto")
+    assert g["status"] == 0
+    compare_rows(g, o)
+    compare_scan(g, o, lay, mode, lam)
