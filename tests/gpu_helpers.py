@@ -17,7 +17,11 @@ Tolerances (stated where the path's outputs are specified):
   the within-turn profile sums: like the per-turn sums; retained-token counts
   and profile counts exact;
 * a stop index may differ from the oracle's only where the oracle's running
-  sum lies within 1e-3 of lambda at every test position between the two.
+  sum lies within 1e-3 of lambda at every test position between the two;
+  with equal stop indices, a token whose oracle running sum before it lies
+  within 1e-3 of lambda may be retained or not (the retained count lies
+  between the prefixes retained for certain and at most; the loss is the
+  certain prefix's plus at most those tokens' terms).
 """
 from __future__ import annotations
 
@@ -165,16 +169,47 @@ def compare_scan(g, o, lay, mode, lam):
         assert bool(st["stopped"][i]) == (gr >= 0)
         assert int(st["rows_seen"][i]) == r1 - r0
         if gr == orr:
-            # OPD loss on the retained tokens (Eq. 2, Algorithm 1)
-            assert int(st["loss_tokens"][i]) == int(o["traj_loss_tokens"][i]), ("loss_tokens", i)
+            # OPD loss on the retained tokens (Eq. 2, Algorithm 1): a token is
+            # retained while the rule has not fired before it, i.e. while the
+            # oracle's running sum before it is >= lambda; the sum never
+            # rises, so the retained tokens are a prefix.  Tokens whose sum
+            # before them lies within TIE_BAND of lambda may be counted
+            # either way (the tie-band rule of stop_matches): the count must
+            # lie between the prefix retained for certain and the prefix
+            # retained at most, the loss must be the certain prefix's plus at
+            # most the tie tokens' terms.  Without a tie both are exact.
+            before = _sum_before(o, lay, mode, i) - lam_a[i]
+            sure, maybe = before >= TIE_BAND, before > -TIE_BAND
+            term = (lp[r0:r1] + d[r0:r1]) * d[r0:r1]
+            n_lo, n_hi = int(sure.sum()), int(maybe.sum())
+            assert n_lo <= int(o["traj_loss_tokens"][i]) <= n_hi  # the oracle's own count
+            assert n_lo <= int(st["loss_tokens"][i]) <= n_hi, ("loss_tokens", i, n_lo, n_hi)
+            l_tie = float(np.abs(term[maybe & ~sure]).sum())
             mag = loss_mag(lp[r0:r1] + d[r0:r1], d[r0:r1])
-            assert abs(st["loss"][i] - o["traj_loss"][i]) <= SUM_RTOL * mag, ("loss", i)
+            assert abs(st["loss"][i] - float(term[sure].sum())) <= SUM_RTOL * mag + l_tie, ("loss", i)
+            if n_lo == n_hi:
+                assert int(st["loss_tokens"][i]) == int(o["traj_loss_tokens"][i]), ("loss_tokens", i)
+                assert abs(st["loss"][i] - o["traj_loss"][i]) <= SUM_RTOL * mag, ("loss", i)
     if "profile" in g:
         # within-turn decile profile (Observation 1): counts exact, sums 1e-5 of magnitudes
         gp, op = g["profile"], o["profile"]
         assert np.array_equal(gp[:, 2], op[:, 2]), (gp[:, 2], op[:, 2])
         assert np.all(np.abs(gp[:, 0] - op[:, 0]) <= SUM_RTOL * (np.sum(np.abs(d)) + len(d))), "profile d"
         assert np.all(np.abs(gp[:, 1] - op[:, 1]) <= SUM_RTOL * np.sum(np.abs(lp) + 1.0)), "profile logp_t"
+
+
+def _sum_before(o, lay, mode, i):
+    """The oracle's running sum before each token of trajectory i: the
+    previous token's (TOKEN_SUM) or the previous turn's end (TURN_MEAN); 0
+    before the trajectory's first token or turn."""
+    base = lay.traj_row_off[0]
+    r0, r1 = lay.traj_row_off[i] - base, lay.traj_row_off[i + 1] - base
+    if mode == oracle.TOKEN_SUM:
+        return np.concatenate([[0.0], o["row_cum"][r0:r1 - 1]])
+    k0, k1 = lay.traj_turn_off[i], lay.traj_turn_off[i + 1]
+    n = np.diff(lay.turn_row_off[k0:k1 + 1])
+    prev = np.concatenate([[0.0], o["turn_cum"][k0:k1 - 1]])
+    return np.repeat(prev, n)
 
 
 def pad_cols(a: np.ndarray, ld: int, fill) -> np.ndarray:
