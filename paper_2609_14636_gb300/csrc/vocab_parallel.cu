@@ -289,33 +289,6 @@ __device__ __forceinline__ int smem_upper_le(const int64_t* a, int n, int64_t r)
   return lo;
 }
 
-// A prefix over tiles with its restart marks (the cluster form's fold of
-// the tiles' aggregates).
-struct PreFlag {
-  double c, st, sd, sl;
-  int flags;
-};
-
-__device__ __forceinline__ PreFlag pre_flag_combine(const PreFlag& a, const PreFlag& b) {
-  PreFlag r;
-  r.c = (b.flags & kRestartSum) ? b.c : a.c + b.c;
-  r.st = (b.flags & kRestartTurn) ? b.st : a.st + b.st;
-  r.sd = (b.flags & kRestartTurn) ? b.sd : a.sd + b.sd;
-  r.sl = (b.flags & kRestartTurn) ? b.sl : a.sl + b.sl;
-  r.flags = a.flags | b.flags;
-  return r;
-}
-
-__device__ __forceinline__ PreFlag pre_flag_shfl(const PreFlag& v, int src) {
-  PreFlag o;
-  o.c = __shfl_sync(0xffffffffu, v.c, src);
-  o.st = __shfl_sync(0xffffffffu, v.st, src);
-  o.sd = __shfl_sync(0xffffffffu, v.sd, src);
-  o.sl = __shfl_sync(0xffffffffu, v.sl, src);
-  o.flags = __shfl_sync(0xffffffffu, v.flags, src);
-  return o;
-}
-
 // The cluster form (CLUSTER; a small window of at most kClusterMaxTiles
 // tiles, launched as ONE thread-block cluster of one CTA per tile, so that
 // the tiles run at once): in place of the lookback through global memory,
@@ -343,7 +316,7 @@ __global__ void __launch_bounds__(TILE) scan_logprobs_tile_kernel(const BatchPar
   __shared__ TileElem s_wpre[kWarps];
   __shared__ TrajElem s_ttot[kWarps];
   __shared__ TrajElem s_tpre[kWarps];
-  __shared__ PreElem s_excl;
+  __shared__ TileElem s_excl;  // the tile's exclusive prefix (flags unused)
   __shared__ TileElem s_agg;
   __shared__ int s_flags;  // bit 0: lookback timed out
   __shared__ double s_prof[3 * STRIDE_PROFILE_BINS];
@@ -465,7 +438,8 @@ __global__ void __launch_bounds__(TILE) scan_logprobs_tile_kernel(const BatchPar
     }
   }
   TileElem x = {0.0, 0.0, 0.0, 0.0, 0};
-  double c_before = 0.0, st_before = 0.0, e_sl = 0.0, ri_c = 0.0;
+  double c_before = 0.0, st_before = 0.0, ri_c = 0.0;
+  float st_before_f = 0.f, e_sl = 0.f;
   if (live) {
     const float nan = __int_as_float(0x7fc00000);
     if (meta.bad) {
@@ -478,23 +452,31 @@ __global__ void __launch_bounds__(TILE) scan_logprobs_tile_kernel(const BatchPar
     const float dd = lps - lpt;
     if (p.out.opd) p.out.opd[w] = dd;
     const int64_t n_k = meta.turn_end - meta.turn_start;
-    const double ec = (p.mode == STRIDE_STOP_TURN_MEAN) ? (double)lpt / (double)(n_k > 0 ? n_k : 1) : (double)lpt;
-    const double est = (double)lpt, esd = (double)dd, esl = (double)lps * (double)dd;
+    // The row's terms in fp32 (logp_S * d rounded once, as the fp64 product
+    // of two floats rounded to float would be); the stop-sum term in fp64,
+    // a turn mean's share lpt / n_k rounded once to fp32 first (GB300 issues
+    // an fp64 divide as a sequence of fp64 operations at 1/64 of the fp32
+    // rate; the rounding is 6e-8 of the term).
+    const float esl = lps * dd;
+    const double ec =
+        (p.mode == STRIDE_STOP_TURN_MEAN) ? (double)(lpt / (float)(n_k > 0 ? n_k : 1)) : (double)lpt;
     e_sl = esl;
     if (p.profile && !meta.bad) {
       const int jb = (int)((10 * (r - meta.turn_start)) / n_k);  // Observation 1 decile
-      atomicAdd(s_prof + 3 * jb + 0, esd);
-      atomicAdd(s_prof + 3 * jb + 1, est);
+      atomicAdd(s_prof + 3 * jb + 0, (double)dd);
+      atomicAdd(s_prof + 3 * jb + 1, (double)lpt);
       atomicAdd(s_prof + 3 * jb + 2, 1.0);
     }
     if (seeded && !meta.bad) {
-      x = TileElem{cum0 + ec, (float)(st0 + est), (float)(sd0 + esd), (float)(sl0 + esl), kRestartSum | kRestartTurn};
+      x = TileElem{cum0 + ec, (float)(st0 + (double)lpt), (float)(sd0 + (double)dd), (float)(sl0 + (double)esl),
+                   kRestartSum | kRestartTurn};
       c_before = cum0;
       st_before = st0;
+      st_before_f = (float)st0;
     } else if (seeded) {
-      x = TileElem{ec, (float)est, (float)esd, (float)esl, kRestartSum | kRestartTurn};  // NaN: nothing after a bad row is meaningful
+      x = TileElem{ec, lpt, dd, esl, kRestartSum | kRestartTurn};  // NaN: nothing after a bad row is meaningful
     } else {
-      x = TileElem{ec, (float)est, (float)esd, (float)esl, fturn ? kRestartTurn : 0};
+      x = TileElem{ec, lpt, dd, esl, fturn ? kRestartTurn : 0};
     }
     if (seeded) x.flags |= 4;  // bit 2: this row's exclusive prefix is the carried state, not the scan
   }
@@ -519,19 +501,17 @@ __global__ void __launch_bounds__(TILE) scan_logprobs_tile_kernel(const BatchPar
     cluster_arrive_release();
     cluster_wait_acquire();  // every aggregate has arrived; nothing touches this CTA's memory after
     if (warp == 0) {
-      PreFlag v = {0.0, 0.0, 0.0, 0.0, 0};
-      if (lane < tile) {
-        const TileElem a = s_caggs[lane];
-        v = PreFlag{a.c, (double)a.st, (double)a.sd, (double)a.sl, a.flags};
-      }
+      // the predecessors' aggregates folded in tile order (a warp scan: the
+      // stop sum fp64, the open-turn sums fp32 as inside a tile)
+      TileElem v = {0.0, 0.f, 0.f, 0.f, 0};
+      if (lane < tile) v = s_caggs[lane];
 #pragma unroll
       for (int d = 1; d < kClusterMaxTiles; d <<= 1) {
-        const PreFlag o = pre_flag_shfl(v, lane >= d ? lane - d : lane);
-        if (lane >= d) v = pre_flag_combine(o, v);
+        const TileElem o = tile_shfl_up(v, d);
+        if (lane >= d) v = tile_combine(o, v);
       }
-      const PreFlag pf = pre_flag_shfl(v, tile > 0 ? (int)tile - 1 : 0);
-      if (lane == 0) {
-        s_excl = tile > 0 ? PreElem{pf.c, pf.st, pf.sd, pf.sl} : PreElem{0.0, 0.0, 0.0, 0.0};
+      if (lane == (tile > 0 ? (int)tile - 1 : 0)) {
+        s_excl = tile > 0 ? TileElem{v.c, v.st, v.sd, v.sl, 0} : TileElem{0.0, 0.f, 0.f, 0.f, 0};
         s_flags = 0;
       }
     }
@@ -564,7 +544,7 @@ __global__ void __launch_bounds__(TILE) scan_logprobs_tile_kernel(const BatchPar
         }
       }
       if (lane == 0) {
-        s_excl = pre;
+        s_excl = TileElem{pre.c, (float)pre.st, (float)pre.sd, (float)pre.sl, 0};
         s_flags = timed_out ? 1 : 0;
       }
     }
@@ -573,16 +553,19 @@ __global__ void __launch_bounds__(TILE) scan_logprobs_tile_kernel(const BatchPar
 
   // 5. complete every row
   if (live) {
-    const PreElem pre = s_excl;
-    const PreElem ri = pre_combine(pre, tile_incl);
+    // the row's prefixes: the stop sum fp64, the open-turn sums fp32 (the
+    // tile's prefix rounded once to fp32; 6e-8 of the sums)
+    const TileElem pre = s_excl;
+    const TileElem ri = tile_combine(pre, tile_incl);
     if (!(x.flags & 4)) {
-      const PreElem re = pre_combine(pre, tile_excl);
+      const TileElem re = tile_combine(pre, tile_excl);
       c_before = re.c;
-      st_before = fturn ? 0.0 : re.st;
+      st_before_f = fturn ? 0.f : re.st;
+      st_before = (double)st_before_f;
     }
     RowCarry rc;
-    rc.e = ScanElem{0.0, 0.0, 0.0, e_sl, fturn};
-    const ScanElem si{ri.c, ri.st, ri.sd, ri.sl, 1};
+    rc.e = ScanElem{0.0, 0.0, 0.0, (double)e_sl, fturn};
+    const ScanElem si{ri.c, (double)ri.st, (double)ri.sd, (double)ri.sl, 1};
     row_tail(p, r, meta, rc, si, c_before, st_before, (s_flags & 1) != 0, true);
     ri_c = ri.c;
   }
@@ -599,9 +582,10 @@ __global__ void __launch_bounds__(TILE) scan_logprobs_tile_kernel(const BatchPar
     const bool turn_last = (r == meta.turn_end - 1);
     const bool test = (p.mode == STRIDE_STOP_TOKEN_SUM) || turn_last;
     cross = test && ri_c < (double)lam;
-    const double before = (p.mode == STRIDE_STOP_TOKEN_SUM) ? c_before : c_before - st_before / (double)n_k;
+    const double before =
+        (p.mode == STRIDE_STOP_TOKEN_SUM) ? c_before : c_before - (double)(st_before_f / (float)n_k);
     const bool kept = before >= (double)lam;
-    te = TrajElem{kept ? (float)e_sl : 0.f, kept ? 1 : 0, cross ? 1 : 0, r == meta.traj_start ? 1 : 0};
+    te = TrajElem{kept ? e_sl : 0.f, kept ? 1 : 0, cross ? 1 : 0, r == meta.traj_start ? 1 : 0};
   }
   const TrajElem traj_id = {0.f, 0, 0, 0};
   TrajElem t_incl, t_excl;
