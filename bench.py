@@ -1190,7 +1190,7 @@ def measure_tiny(args, dev, local, ws=1) -> dict:
                      "frac": bpr * R / (ms * 1e-3) / 1e9 / peak, "traffic": None,
                      "algorithmic_bytes_per_launch": bpr * R,
                      "kernel": "score_batch_split_kernel<f32> (2-CTA clusters, one wave of 1,024 CTAs) "
-                               "+ scan_logprobs_tile_kernel (4 tiles of 128 rows)",
+                               "+ scan_logprobs_tile_kernel (4 tiles of 128 rows, one 4-CTA cluster)",
                      "note": "512 rows on 152 SMs: a latency-bound launch; time includes state init",
                      "ms_per_step_write_flush_only": ms_write_only,
                      "frac_write_flush_only": bpr * R / (ms_write_only * 1e-3) / 1e9 / peak},
