@@ -355,8 +355,15 @@ __global__ void __launch_bounds__(TILE) scan_logprobs_tile_kernel(const BatchPar
   }
 
   // 1. the tile's first turn (warp 0) and first trajectory (warp 1), then
-  //    the offsets of the next TILE + 1 of each in shared memory
-  if (warp == 0) {
+  //    the offsets of the next TILE + 1 of each in shared memory (a layout
+  //    of at most TILE turns and trajectories: all of them, no search --
+  //    one dependent round trip less before the wait)
+  if (p.n_turns <= TILE && p.n_traj <= TILE) {
+    if (tid == 0) {
+      s_first[0] = p.n_turns > 0 ? 0 : -1;
+      s_first[1] = 0;
+    }
+  } else if (warp == 0) {
     const bool ok = p.n_turns > 0 && __ldg(p.turn_row_off) <= r0;
     const int64_t k0 = ok ? warp_upper_le(p.turn_row_off, 0, p.n_turns - 1, r0, lane) : 0;
     if (lane == 0) s_first[0] = ok ? k0 : -1;
