@@ -39,16 +39,16 @@
  * - Errors found on the device are OR-ed into the caller's int32 `dev_status`
  *   word (STRIDE_DEV_* bits; nullable), readable after the stream has
  *   synchronised.  Kernels never trap: a bad row gets NaN outputs.
- * - Logit rows are row-major with a row stride `ld` (elements, ld >= V).
+ * - Logit rows are row-major with a row stride `ld` (elements, ld >= V), and
+ *   1 <= V <= STRIDE_MAX_VOCAB (for a vocabulary shard, its V_shard).
  *   Rows whose address and stride are 16-byte aligned take the vectorised
  *   path; others take a scalar path with the same results.
  * - Turn and row indices reported per trajectory are 0-based and local to the
  *   trajectory.  The paper's turns are 1-based, so the returned k* equals its
  *   K0 = k* - 1 (Algorithm 1): the number of turns reused as context.
- * - Every compute call is a plain kernel launch or two (plus a
- *   cudaMemsetAsync of the workspace on the batch paths other than the
- *   small-window one), so a sequence of calls can be captured in a CUDA
- *   graph.
+ * - Every compute call is a plain kernel launch or a short chain of them
+ *   (the batch paths clear their workspace with a kernel of the chain), so
+ *   a sequence of calls can be captured in a CUDA graph.
  * - The library is built for sm_103a only; on another device the calls return
  *   STRIDE_ERR_UNSUPPORTED_DEVICE.  There is no CPU fallback.
  * - The batch calls choose among three kernels with the same results: for
@@ -98,6 +98,12 @@ typedef enum stride_status {
 /* ---- enums ---------------------------------------------------------------- */
 #define STRIDE_DTYPE_BF16 0 /* logits are bfloat16 */
 #define STRIDE_DTYPE_F32 1  /* logits are float32 */
+
+/* The largest vocabulary (logits per row, or per shard row) the scoring
+ * calls accept.  The kernels index a row's columns with 32-bit integers;
+ * 2^30 keeps every column index plus a CTA's stride below 2^31.  A larger
+ * V (or V_shard) returns STRIDE_ERR_INVALID_ARG before any launch. */
+#define STRIDE_MAX_VOCAB (1 << 30)
 
 #define STRIDE_STOP_TURN_MEAN 0 /* Eq. 5: running sum of per-turn means l_k, tested at turn ends */
 #define STRIDE_STOP_TOKEN_SUM 1 /* Sec. 5.5: running sum of token log-probs, tested at every token */

@@ -40,6 +40,7 @@ TURN_MEAN, TOKEN_SUM = 0, 1
 DEV_TOKEN_RANGE, DEV_BAD_LAYOUT, DEV_TIMEOUT = 0x1, 0x2, 0x4
 ROW_OUTPUT_KEYS = ("logp_s", "logp_t", "opd", "lse_s", "lse_t", "x_s", "x_t")
 NOALLOC_MAX_ROWS = 65536  # STRIDE_NOALLOC_MAX_ROWS
+MAX_VOCAB = 1 << 30  # STRIDE_MAX_VOCAB
 OK, ERR_INVALID_ARG, ERR_UNSUPPORTED_DTYPE, ERR_WORKSPACE, ERR_CUDA, ERR_UNSUPPORTED_DEVICE, ERR_TOO_LARGE = range(7)
 
 STATE_DTYPE = np.dtype([("cum", "<f8"), ("turn_sum_t", "<f8"), ("turn_sum_d", "<f8"),

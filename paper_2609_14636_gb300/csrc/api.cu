@@ -41,7 +41,7 @@ bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) ==
 int check_logits(const void* S, const void* T, int32_t dtype, int64_t ld, int64_t V) {
   if (dtype_bytes(dtype) == 0) return STRIDE_ERR_UNSUPPORTED_DTYPE;
   if (!S || !T) return STRIDE_ERR_INVALID_ARG;
-  if (V < 1 || V > INT32_MAX || ld < V) return STRIDE_ERR_INVALID_ARG;
+  if (V < 1 || V > STRIDE_MAX_VOCAB || ld < V) return STRIDE_ERR_INVALID_ARG;
   return STRIDE_OK;
 }
 

@@ -49,3 +49,11 @@ def test_header_compiles_as_c():
                        input='#include "stride.h"\n#include "stride_selftest.h"\nint main(void){return sizeof(stride_scan_state)==80 && sizeof(stride_turn_stats)==40 ? 0 : 1;}\n',
                        capture_output=True, text=True)
     assert r.returncode == 0, r.stderr
+
+
+def test_max_vocab_constant_matches_header():
+    import paper_2609_14636_gb300 as stride
+
+    src = (ROOT / "include" / "stride.h").read_text()
+    m = re.search(r"#define STRIDE_MAX_VOCAB \(1 << (\d+)\)", src)
+    assert m and stride.MAX_VOCAB == 1 << int(m.group(1)) == 1 << 30
