@@ -123,8 +123,10 @@ __global__ void __launch_bounds__(kBatchThreads, 2) score_batch_kernel(const Bat
 // the tiled scan on those log-probs (vocab_parallel.cu), launched as a
 // programmatic dependent of this kernel.  In a window whose rows all finish
 // streaming together, a lookback per row cost a chain of prefixes after the
-// last row (12 us on a 512-row segment); the tiled scan folds 256 rows per
-// step of that chain.
+// last row (12 us on a 512-row segment); the tiled scan scans 128 rows per
+// CTA, and a window of at most 16 such tiles runs as one cluster whose
+// tiles exchange their aggregates through distributed shared memory (no
+// chain at all).
 namespace cg = cooperative_groups;
 constexpr int kSplitMaxCluster = 8;
 constexpr int kSplitThreads = 128;

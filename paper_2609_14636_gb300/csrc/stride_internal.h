@@ -28,7 +28,8 @@ constexpr int kFlagStride = 32;
 // on GB300 (one size for both): the 148,909-row scan took 52.8 / 51.2 / 49.2
 // / 49.6 us with tiles of 64 / 128 / 256 / 512 rows, the 512-row tiny step
 // 36.6 / 36.7 / 37.4 / 39.0 us: many small tiles finish a small window's
-// chain sooner, larger ones run a long scan with fewer lookbacks.
+// chain sooner, larger ones run a long scan with fewer lookbacks.  (The
+// small window's tiles now run as one cluster, with no chain.)
 #ifndef STRIDE_SCAN_TILE_ROWS
 #define STRIDE_SCAN_TILE_ROWS 256
 #endif
@@ -136,8 +137,8 @@ int current_device_sms(int* dev_out, cudaError_t* err);
 
 // Launchers return a cudaError_t from the launch.
 // Clears what must start at zero in the workspace (clear_bytes from its
-// start: a memset, or on the small-window path the kernel itself) and
-// launches the batch scoring kernels.
+// start: the clearing kernel, or on the small-window path the split kernel
+// itself) and launches the batch scoring kernels.
 cudaError_t launch_score_batch(const BatchParams& p, int dtype, bool vec, size_t clear_bytes, cudaStream_t stream);
 cudaError_t launch_score_batch_stream(const BatchParams& p, int dtype, cudaStream_t stream);
 // Zeroes `bytes` (a multiple of 16) at ws as a programmatic dependent of the
