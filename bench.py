@@ -262,6 +262,9 @@ def main() -> None:
     ap.add_argument("--rows-list", default="8,16,32,48,64,96,128,160,192,224,256", help="step_shapes: live rows")
     ap.add_argument("--shapes", default="0x0,128x4,128x6,128x8,128x12,128x16,512x4,512x8",
                     help="step_shapes: CTA threads x CTAs per row (0x0 = automatic)")
+    ap.add_argument("--step-shape", default="",
+                    help="decode_step: a fixed launch shape THREADSxCLUSTER for every step "
+                         "(stride_force_step_shape), for comparisons; default: the library's choice")
     ap.add_argument("--max-rows", type=int, default=0,
                     help="score only the leading whole trajectories that fit (small profiling cases)")
     args = ap.parse_args()
@@ -879,7 +882,19 @@ def run_decode(args) -> None:
     stopped rollouts masked).  Also a 64-step all-active graph (lambda =
     -inf), which shows the kernel at full activity."""
     ws, rank, local, dev = _setup_rank()
-    line = measure_decode(args, dev, local, ws)
+    shape = getattr(args, "step_shape", "")
+    if shape:
+        import paper_2609_14636_gb300 as stride
+
+        th, C = (int(v) for v in shape.split("x"))
+        stride.stride_force_step_shape(th, C)
+    try:
+        line = measure_decode(args, dev, local, ws)
+    finally:
+        if shape:
+            stride.stride_force_step_shape(0, 0)
+    if shape:
+        line["config"]["forced_step_shape"] = shape
     if rank == 0:
         print(json.dumps(line), flush=True)
 
