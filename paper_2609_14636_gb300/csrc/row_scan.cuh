@@ -306,9 +306,12 @@ __device__ __forceinline__ RowCarry row_finalize(const BatchParams& p, int64_t t
 // row's OPD-loss term if the row is retained, and the carried state.
 //
 // Retention: a row is retained when the stop rule has not fired before it.
-// In token mode that is "the running sum before the row is >= lambda"; in
-// turn mode "the running sum through the previous turn is >= lambda", which
-// is the running sum before the row minus the row's turn's terms so far
+// A trajectory's first token (token mode) or first turn (turn mode) always
+// is: no test precedes it (with a prefix-buffer offset already below lambda
+// that token or turn triggers the stop and is kept).  After it, in token
+// mode that is "the running sum before the row is >= lambda"; in turn mode
+// "the running sum through the previous turn is >= lambda", which is the
+// running sum before the row minus the row's turn's terms so far
 // (c_before - st_before / n_k).  The sums are monotone, so this selects
 // exactly the rows up to the first crossing (its turn, in turn mode).
 // rc is read in lane 0.
@@ -370,8 +373,9 @@ __device__ __forceinline__ void row_tail(const BatchParams& p, int64_t r, const 
       atomicMin(reinterpret_cast<unsigned int*>(&sp->stop_turn), (unsigned int)meta.local_turn);
       sp->stopped = 1;
     }
+    const bool first = (p.mode == STRIDE_STOP_TOKEN_SUM) ? (r == meta.traj_start) : (meta.local_turn == 0);
     const double before = (p.mode == STRIDE_STOP_TOKEN_SUM) ? c_before : c_before - st_before / (double)n_k;
-    if (before >= (double)lam) {
+    if (first || before >= (double)lam) {
       atomicAdd(&sp->loss, rc.e.sl);
       atomicAdd(reinterpret_cast<unsigned long long*>(&sp->loss_tokens), 1ull);
     }

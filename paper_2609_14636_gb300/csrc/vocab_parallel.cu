@@ -589,9 +589,12 @@ __global__ void __launch_bounds__(TILE) scan_logprobs_tile_kernel(const BatchPar
     const bool turn_last = (r == meta.turn_end - 1);
     const bool test = (p.mode == STRIDE_STOP_TOKEN_SUM) || turn_last;
     cross = test && ri_c < (double)lam;
+    // retained unless the rule fired before the row (row_tail); a
+    // trajectory's first token or turn always is
+    const bool first = (p.mode == STRIDE_STOP_TOKEN_SUM) ? (r == meta.traj_start) : (meta.local_turn == 0);
     const double before =
         (p.mode == STRIDE_STOP_TOKEN_SUM) ? c_before : c_before - (double)(st_before_f / (float)n_k);
-    const bool kept = before >= (double)lam;
+    const bool kept = first || before >= (double)lam;
     te = TrajElem{kept ? e_sl : 0.f, kept ? 1 : 0, cross ? 1 : 0, r == meta.traj_start ? 1 : 0};
   }
   const TrajElem traj_id = {0.f, 0, 0, 0};

@@ -170,16 +170,20 @@ def compare_scan(g, o, lay, mode, lam):
         assert int(st["rows_seen"][i]) == r1 - r0
         if gr == orr:
             # OPD loss on the retained tokens (Eq. 2, Algorithm 1): a token is
-            # retained while the rule has not fired before it, i.e. while the
-            # oracle's running sum before it is >= lambda; the sum never
+            # retained while the rule has not fired before it -- the
+            # trajectory's first token (token mode) or first turn (turn mode)
+            # always, no test preceding it; after it, while the oracle's
+            # running sum at the previous test is >= lambda.  The sum never
             # rises, so the retained tokens are a prefix.  Tokens whose sum
             # before them lies within TIE_BAND of lambda may be counted
             # either way (the tie-band rule of stop_matches): the count must
             # lie between the prefix retained for certain and the prefix
             # retained at most, the loss must be the certain prefix's plus at
             # most the tie tokens' terms.  Without a tie both are exact.
-            before = _sum_before(o, lay, mode, i) - lam_a[i]
-            sure, maybe = before >= TIE_BAND, before > -TIE_BAND
+            before, first = _sum_before(o, lay, mode, i)
+            with np.errstate(invalid="ignore"):
+                gap = before - lam_a[i]
+            sure, maybe = first | (gap >= TIE_BAND), first | (gap > -TIE_BAND)
             term = (lp[r0:r1] + d[r0:r1]) * d[r0:r1]
             n_lo, n_hi = int(sure.sum()), int(maybe.sum())
             assert n_lo <= int(o["traj_loss_tokens"][i]) <= n_hi  # the oracle's own count
@@ -199,17 +203,22 @@ def compare_scan(g, o, lay, mode, lam):
 
 
 def _sum_before(o, lay, mode, i):
-    """The oracle's running sum before each token of trajectory i: the
-    previous token's (TOKEN_SUM) or the previous turn's end (TURN_MEAN); 0
-    before the trajectory's first token or turn."""
+    """The oracle's running sum at the last test before each token of
+    trajectory i: the previous token's (TOKEN_SUM) or the previous turn's
+    end (TURN_MEAN); and the mask of the tokens no test precedes (the first
+    token, or the first turn's tokens), whose entry is 0."""
     base = lay.traj_row_off[0]
     r0, r1 = lay.traj_row_off[i] - base, lay.traj_row_off[i + 1] - base
     if mode == oracle.TOKEN_SUM:
-        return np.concatenate([[0.0], o["row_cum"][r0:r1 - 1]])
+        before = np.concatenate([[0.0], o["row_cum"][r0:r1 - 1]])
+        first = np.zeros(r1 - r0, bool)
+        first[0] = True
+        return before, first
     k0, k1 = lay.traj_turn_off[i], lay.traj_turn_off[i + 1]
     n = np.diff(lay.turn_row_off[k0:k1 + 1])
     prev = np.concatenate([[0.0], o["turn_cum"][k0:k1 - 1]])
-    return np.repeat(prev, n)
+    first = np.repeat(np.arange(k1 - k0) == 0, n)
+    return np.repeat(prev, n), first
 
 
 def pad_cols(a: np.ndarray, ld: int, fill) -> np.ndarray:

@@ -107,3 +107,25 @@ def test_no_tie_trajectory_is_exact():
     _drop_rows(g, o, lay, 1, [0])
     with pytest.raises(AssertionError):
         compare_scan(g, o, lay, oracle.TURN_MEAN, lam)
+
+
+@pytest.mark.parametrize("mode", [oracle.TURN_MEAN, oracle.TOKEN_SUM])
+def test_first_test_is_always_retained(mode):
+    """lambda = +inf: the rule fires at the first test, after the first turn
+    (or token), which is retained -- the comparison must demand it."""
+    lay = synth.layout_from_turn_lengths(TURNS)
+    rng = np.random.default_rng(7)
+    R = lay.rows
+    lpt = -rng.integers(1, 9, R).astype(np.float64) * 0.25
+    d = rng.integers(-4, 5, R).astype(np.float64) * 0.125
+    lps = lpt + d
+    lam = np.array([np.inf, -np.inf])
+    o = oracle.scan_batch(lpt, d, lay.traj_row_off, lay.turn_row_off, lay.traj_turn_off, mode, lam, logp_s=lps)
+    o.update(logp_t=lpt, logp_s=lps, d=d)
+    kept = TURNS[0][0] if mode == oracle.TURN_MEAN else 1
+    assert o["traj_loss_tokens"][0] == kept and o["traj_loss_tokens"][1] == sum(TURNS[1])
+    compare_scan(_as_gpu(o, lay), o, lay, mode, lam)
+    g = _as_gpu(o, lay)
+    _drop_rows(g, o, lay, 0, range(kept))
+    with pytest.raises(AssertionError):
+        compare_scan(g, o, lay, mode, lam)

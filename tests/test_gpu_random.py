@@ -194,3 +194,43 @@ def test_small_window_scan_every_cluster_size(stride, rows, mode):
     assert g["status"] == 0
     compare_rows(g, o)
     compare_scan(g, o, lay, mode, lam)
+
+
+@pytest.mark.parametrize("kernel", ["auto", "stream", "split", "rows"])
+@pytest.mark.parametrize("mode", [0, 1])
+@pytest.mark.parametrize("lam", [float("inf"), float("-inf")])
+def test_infinite_thresholds(stride, kernel, mode, lam):
+    """lambda = +inf: every trajectory stops at its first test (its first
+    turn's end, or its first token) and keeps exactly that turn or token;
+    lambda = -inf: none stops and every token is retained -- in one window
+    and in three windows with the carried state."""
+    rng = np.random.default_rng(777 + mode)
+    lens = [[1 if rng.random() < 0.2 else int(rng.integers(2, 90)) for _ in range(int(rng.integers(1, 5)))]
+            for _ in range(6)]
+    lay = synth.layout_from_turn_lengths(lens)
+    R, V = lay.rows, 1000
+    S = rng.standard_normal((R, V), dtype=np.float32) * np.float32(2.0)
+    T = S + rng.standard_normal((R, V), dtype=np.float32)
+    tok = rng.integers(0, V, R).astype(np.int32)
+    o = oracle_batch(S, T, tok, lay, mode, np.float32(lam))
+    # the definitions' answer, independent of the oracle
+    first = np.diff(lay.turn_row_off)[lay.traj_turn_off[:-1]]
+    if lam > 0:
+        want_row = np.zeros(lay.n_traj, np.int64) if mode == 1 else first - 1
+        assert np.array_equal(o["stop_row"], want_row) and np.all(o["stop_turn"] == 0)
+        assert np.array_equal(o["traj_loss_tokens"], want_row + 1)
+    else:
+        assert np.all(o["stop_row"] == -1)
+        assert np.array_equal(o["traj_loss_tokens"], np.diff(lay.traj_row_off))
+    cuts = [0, R // 3, (2 * R) // 3, R]
+    stride.stride_force_batch_kernel(kernel)
+    try:
+        for windows in (None, list(zip(cuts[:-1], cuts[1:]))):
+            g = run_batch(stride, S, T, tok, lay, mode, np.float32(lam), windows=windows, V=V)
+            assert g["status"] == 0
+            compare_rows(g, o)
+            compare_scan(g, o, lay, mode, np.float32(lam))
+            assert np.array_equal(g["state"]["stop_row"], o["stop_row"])
+            assert np.array_equal(g["state"]["loss_tokens"], o["traj_loss_tokens"])
+    finally:
+        stride.stride_force_batch_kernel("auto")
