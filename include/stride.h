@@ -189,9 +189,12 @@ STRIDE_API size_t stride_score_batch_workspace_size(int64_t window_rows);
  * stop_mode: STRIDE_STOP_TURN_MEAN or STRIDE_STOP_TOKEN_SUM.  lambda: device
  * float [n_traj] per-trajectory thresholds, or NULL to use lambda_all for
  * every trajectory (the scale of lambda depends on the generation unit and is
- * chosen per domain, Sec. 4.1).  The test is strict: sum < lambda.  The
- * token or turn that triggers is retained (Sec. 4.1).  Later turns are still
- * scored; the stop fields keep the first crossing.
+ * chosen per domain, Sec. 4.1).  The test is strict: sum < lambda (a NaN
+ * entry of the array never fires: nothing stops and every token is
+ * retained; a NaN lambda_all is rejected).  The token or turn that triggers
+ * is retained (Sec. 4.1), and so is a trajectory's first turn or token
+ * whatever its starting sum.  Later turns are still scored; the stop fields
+ * keep the first crossing.
  *
  * state: device [n_traj], in/out (see stride_scan_state).
  * out: host struct of optional per-row outputs indexed by (row - row_begin); NULL for none.

@@ -375,7 +375,7 @@ __device__ __forceinline__ void row_tail(const BatchParams& p, int64_t r, const 
     }
     const bool first = (p.mode == STRIDE_STOP_TOKEN_SUM) ? (r == meta.traj_start) : (meta.local_turn == 0);
     const double before = (p.mode == STRIDE_STOP_TOKEN_SUM) ? c_before : c_before - st_before / (double)n_k;
-    if (first || before >= (double)lam) {
+    if (first || !(before < (double)lam)) {  // the previous test did not fire (a NaN lambda never does)
       atomicAdd(&sp->loss, rc.e.sl);
       atomicAdd(reinterpret_cast<unsigned long long*>(&sp->loss_tokens), 1ull);
     }

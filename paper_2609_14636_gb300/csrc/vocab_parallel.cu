@@ -594,7 +594,7 @@ __global__ void __launch_bounds__(TILE) scan_logprobs_tile_kernel(const BatchPar
     const bool first = (p.mode == STRIDE_STOP_TOKEN_SUM) ? (r == meta.traj_start) : (meta.local_turn == 0);
     const double before =
         (p.mode == STRIDE_STOP_TOKEN_SUM) ? c_before : c_before - (double)(st_before_f / (float)n_k);
-    const bool kept = first || before >= (double)lam;
+    const bool kept = first || !(before < (double)lam);
     te = TrajElem{kept ? e_sl : 0.f, kept ? 1 : 0, cross ? 1 : 0, r == meta.traj_start ? 1 : 0};
   }
   const TrajElem traj_id = {0.f, 0, 0, 0};

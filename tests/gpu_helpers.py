@@ -183,7 +183,9 @@ def compare_scan(g, o, lay, mode, lam):
             before, first = _sum_before(o, lay, mode, i)
             with np.errstate(invalid="ignore"):
                 gap = before - lam_a[i]
-            sure, maybe = first | (gap >= TIE_BAND), first | (gap > -TIE_BAND)
+            # (a NaN lambda never fires: every token retained)
+            sure = first | (gap >= TIE_BAND) | bool(np.isnan(lam_a[i]))
+            maybe = sure | (gap > -TIE_BAND)
             term = (lp[r0:r1] + d[r0:r1]) * d[r0:r1]
             n_lo, n_hi = int(sure.sum()), int(maybe.sum())
             assert n_lo <= int(o["traj_loss_tokens"][i]) <= n_hi  # the oracle's own count

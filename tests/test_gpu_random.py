@@ -234,3 +234,34 @@ def test_infinite_thresholds(stride, kernel, mode, lam):
             assert np.array_equal(g["state"]["loss_tokens"], o["traj_loss_tokens"])
     finally:
         stride.stride_force_batch_kernel("auto")
+
+
+@pytest.mark.parametrize("kernel", ["auto", "stream", "split", "rows"])
+@pytest.mark.parametrize("mode", [0, 1])
+def test_nan_thresholds_never_fire(stride, kernel, mode):
+    """A NaN entry of the per-trajectory lambda array never fires (the test
+    is strict, sum < lambda): its trajectory never stops and keeps every
+    token, while the finite entries beside it stop as usual."""
+    rng = np.random.default_rng(991 + mode)
+    lens = [[int(rng.integers(2, 60)) for _ in range(int(rng.integers(2, 6)))] for _ in range(8)]
+    lay = synth.layout_from_turn_lengths(lens)
+    R, V = lay.rows, 1000
+    S = rng.standard_normal((R, V), dtype=np.float32) * np.float32(2.0)
+    T = S + rng.standard_normal((R, V), dtype=np.float32)
+    tok = rng.integers(0, V, R).astype(np.int32)
+    o0 = oracle_batch(S, T, tok, lay, mode, np.float32(-1e30))
+    lam = _lambda(o0, lay, mode, rng)
+    lam[::2] = np.float32(np.nan)
+    o = oracle_batch(S, T, tok, lay, mode, lam)
+    assert np.all(o["stop_row"][::2] == -1)
+    assert np.array_equal(o["traj_loss_tokens"][::2], np.diff(lay.traj_row_off)[::2])
+    stride.stride_force_batch_kernel(kernel)
+    try:
+        for windows in (None, [(0, R // 2), (R // 2, R)]):
+            g = run_batch(stride, S, T, tok, lay, mode, lam, windows=windows, V=V)
+            assert g["status"] == 0
+            compare_rows(g, o)
+            compare_scan(g, o, lay, mode, lam)
+            assert np.array_equal(g["state"]["loss_tokens"][::2], np.diff(lay.traj_row_off)[::2])
+    finally:
+        stride.stride_force_batch_kernel("auto")
