@@ -55,7 +55,7 @@ def run_steps(stride, St, Tt, tk, turn_end, ring, B, mode, lam, V, o_rows, form=
     steps = turn_end.shape[0]
     lam32 = np.asarray(lam, np.float32)
     lam64 = np.broadcast_to(lam32.astype(np.float64), (B,))
-    lam_arg = torch.from_numpy(np.ascontiguousarray(np.broadcast_to(lam32, (B,)))).cuda() if lam32.ndim else float(lam32)
+    lam_arg = torch.from_numpy(np.array(np.broadcast_to(lam32, (B,)))).cuda() if lam32.ndim else float(lam32)
     st = stride.new_state(B)
     ost, shadow = oracle.new_rollouts(B), oracle.new_rollouts(B)
     ov, sv = oracle.rollouts_view(ost), oracle.rollouts_view(shadow)
@@ -197,6 +197,26 @@ def test_steps_compact_per_rollout_lambda(stride):
     tk = torch.from_numpy(tok).cuda()
     r = run_steps(stride, St, Tt, tk, turn_end, ring, B, 0, lam, V, o_rows, form="compact")
     assert 0 < r["stopped"] < B
+
+
+@pytest.mark.parametrize("form", ["masked", "compact"])
+def test_steps_nan_thresholds_never_fire(stride, form):
+    """A NaN entry of the per-rollout lambda never fires (the test is
+    strict): that rollout never stops and every token it scores is
+    retained, beside rollouts with finite thresholds that stop as usual."""
+    import torch
+
+    ring, B, steps, V = 3, 24, 160, 4099
+    S, T, tok, Sp, Tp = _ring(78, ring, B, V, V)
+    o_rows = oracle.row_logprobs(S, T, tok)
+    rng = np.random.default_rng(6)
+    turn_end = (rng.random((steps, B)) < 1 / 16).astype(np.uint8)
+    lam = (-24.0 + rng.uniform(-8.0, 8.0, B)).astype(np.float32)
+    lam[::3] = np.float32(np.nan)
+    St, Tt = to_dev(Sp), to_dev(Tp)
+    tk = torch.from_numpy(tok).cuda()
+    r = run_steps(stride, St, Tt, tk, turn_end, ring, B, 0, lam, V, o_rows, form=form)
+    assert 0 < r["stopped"] <= B - len(lam[::3])
 
 
 @pytest.mark.parametrize("threads,C", [(128, 1), (128, 2), (128, 3), (128, 5), (128, 8), (128, 12), (128, 16),
