@@ -265,3 +265,52 @@ def test_nan_thresholds_never_fire(stride, kernel, mode):
             assert np.array_equal(g["state"]["loss_tokens"][::2], np.diff(lay.traj_row_off)[::2])
     finally:
         stride.stride_force_batch_kernel("auto")
+
+
+@pytest.mark.parametrize("kernel", ["auto", "stream", "split", "rows"])
+@pytest.mark.parametrize("mode", [0, 1])
+def test_starting_sums_below_and_above_lambda(stride, kernel, mode):
+    """Running sums that start from a carried offset (the prefix-buffer
+    restart, Sec. 4.1, expressed through the state's cum): where the offset
+    is already below lambda the first test fires and the first turn (or
+    token) is retained; elsewhere the rule runs as usual -- against the
+    oracle given the same starting sums."""
+    import torch
+
+    import oracle
+
+    rng = np.random.default_rng(515 + mode)
+    lens = [[int(rng.integers(2, 50)) for _ in range(int(rng.integers(2, 6)))] for _ in range(8)]
+    lay = synth.layout_from_turn_lengths(lens)
+    R, V = lay.rows, 1000
+    S = rng.standard_normal((R, V), dtype=np.float32) * np.float32(2.0)
+    T = S + rng.standard_normal((R, V), dtype=np.float32)
+    tok = rng.integers(0, V, R).astype(np.int32)
+    lam = np.float32(-40.0 if mode == 0 else -300.0)
+    cum0 = np.where(np.arange(lay.n_traj) % 2 == 0, float(lam) - 5.0, 0.0)  # even: below lambda already
+    o = oracle_batch(S, T, tok, lay, mode, lam)
+    sc = oracle.scan_batch(o["logp_t"], o["d"], lay.traj_row_off, lay.turn_row_off, lay.traj_turn_off, mode,
+                           np.float64(lam), cum_in=cum0, logp_s=o["logp_s"])
+    o.update(sc)
+    first = np.diff(lay.turn_row_off)[lay.traj_turn_off[:-1]]
+    want_row = np.zeros(lay.n_traj, np.int64) if mode == 1 else first - 1
+    assert np.array_equal(o["stop_row"][::2], want_row[::2])
+    assert np.array_equal(o["traj_loss_tokens"][::2], want_row[::2] + 1)
+
+    def seeded():
+        st = stride.new_state(lay.n_traj)
+        h = stride.state_to_numpy(st)[: lay.n_traj].copy()
+        h["cum"] = cum0
+        st[: lay.n_traj].copy_(torch.from_numpy(h.view(np.uint8).reshape(lay.n_traj, -1)).cuda())
+        return st
+
+    stride.stride_force_batch_kernel(kernel)
+    try:
+        for windows in (None, [(0, R // 2), (R // 2, R)]):
+            g = run_batch(stride, S, T, tok, lay, mode, lam, windows=windows, V=V, state=seeded())
+            assert g["status"] == 0
+            compare_scan(g, o, lay, mode, lam)
+            assert np.array_equal(g["state"]["stop_row"][::2], want_row[::2])
+            assert np.array_equal(g["state"]["loss_tokens"][::2], want_row[::2] + 1)
+    finally:
+        stride.stride_force_batch_kernel("auto")
