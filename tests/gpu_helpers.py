@@ -211,6 +211,8 @@ def _sum_before(o, lay, mode, i):
     token, or the first turn's tokens), whose entry is 0."""
     base = lay.traj_row_off[0]
     r0, r1 = lay.traj_row_off[i] - base, lay.traj_row_off[i + 1] - base
+    if r1 == r0:  # a trajectory without turns
+        return np.zeros(0), np.zeros(0, bool)
     if mode == oracle.TOKEN_SUM:
         before = np.concatenate([[0.0], o["row_cum"][r0:r1 - 1]])
         first = np.zeros(r1 - r0, bool)

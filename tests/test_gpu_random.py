@@ -71,6 +71,9 @@ def _lambda(o, lay, mode, rng):
             vals = o["row_cum"][r0:r1]
         else:
             vals = o["turn_cum"][lay.traj_turn_off[i]:lay.traj_turn_off[i + 1]]
+        if len(vals) == 0:  # a trajectory without turns: nothing to test
+            lam[i] = np.float32(-1e6)
+            continue
         if rng.random() < 0.5 or len(vals) == 1:
             lam[i] = np.float32(vals[-1] - 1.0)  # never crosses
         else:
@@ -312,5 +315,41 @@ def test_starting_sums_below_and_above_lambda(stride, kernel, mode):
             compare_scan(g, o, lay, mode, lam)
             assert np.array_equal(g["state"]["stop_row"][::2], want_row[::2])
             assert np.array_equal(g["state"]["loss_tokens"][::2], want_row[::2] + 1)
+    finally:
+        stride.stride_force_batch_kernel("auto")
+
+
+@pytest.mark.parametrize("kernel", ["auto", "stream", "split", "rows"])
+@pytest.mark.parametrize("mode", [0, 1])
+def test_trajectories_without_turns(stride, kernel, mode):
+    """Trajectories with no turns (no rows) among the others -- at the start,
+    between, at the end, and a run of 300 of them (more than one tile of the
+    tiled scan stages) -- are left as initialised, and the rows around them
+    are scored as if they were not there."""
+    rng = np.random.default_rng(808 + mode)
+    lens = [[], []]
+    for k in range(10):
+        lens.append([1 if rng.random() < 0.2 else int(rng.integers(2, 70)) for _ in range(int(rng.integers(1, 5)))])
+        lens.extend([[]] * (300 if k == 4 else int(rng.integers(0, 3))))
+    lens.extend([[], []])
+    lay = synth.layout_from_turn_lengths(lens)
+    R, V = lay.rows, 1000
+    S = rng.standard_normal((R, V), dtype=np.float32) * np.float32(2.0)
+    T = S + rng.standard_normal((R, V), dtype=np.float32)
+    tok = rng.integers(0, V, R).astype(np.int32)
+    o0 = oracle_batch(S, T, tok, lay, mode, np.float32(-1e30))
+    lam = _lambda(o0, lay, mode, np.random.default_rng(9))
+    o = oracle_batch(S, T, tok, lay, mode, lam)
+    empty = np.diff(lay.traj_row_off) == 0
+    stride.stride_force_batch_kernel(kernel)
+    try:
+        for windows in (None, [(0, R // 3), (R // 3, R)]):
+            g = run_batch(stride, S, T, tok, lay, mode, lam, windows=windows, V=V)
+            assert g["status"] == 0
+            compare_rows(g, o)
+            compare_scan(g, o, lay, mode, lam)
+            st = g["state"]
+            assert np.all(st["stop_row"][empty] == -1) and np.all(st["rows_seen"][empty] == 0)
+            assert np.all(st["cum"][empty] == 0.0) and np.all(st["loss_tokens"][empty] == 0)
     finally:
         stride.stride_force_batch_kernel("auto")
