@@ -353,3 +353,32 @@ def test_trajectories_without_turns(stride, kernel, mode):
             assert np.all(st["cum"][empty] == 0.0) and np.all(st["loss_tokens"][empty] == 0)
     finally:
         stride.stride_force_batch_kernel("auto")
+
+
+@pytest.mark.parametrize("kernel", ["auto", "stream", "split", "rows"])
+@pytest.mark.parametrize("width", [1, 2, 3])
+def test_tiny_windows(stride, kernel, width):
+    """Windows of 1-3 rows: nearly every turn, and every trajectory but the
+    shortest, crosses window edges, so the running sum and the open turn's
+    sums go through the carried state at almost every row."""
+    rng = np.random.default_rng(31 + width)
+    lens = [[1 if rng.random() < 0.25 else int(rng.integers(2, 9)) for _ in range(int(rng.integers(1, 4)))]
+            for _ in range(5)]
+    lay = synth.layout_from_turn_lengths(lens)
+    R, V = lay.rows, 300
+    S = rng.standard_normal((R, V), dtype=np.float32) * np.float32(2.0)
+    T = S + rng.standard_normal((R, V), dtype=np.float32)
+    tok = rng.integers(0, V, R).astype(np.int32)
+    for mode in (0, 1):
+        o0 = oracle_batch(S, T, tok, lay, mode, np.float32(-1e30))
+        lam = _lambda(o0, lay, mode, np.random.default_rng(3))
+        o = oracle_batch(S, T, tok, lay, mode, lam)
+        windows = [(a, min(R, a + width)) for a in range(0, R, width)]
+        stride.stride_force_batch_kernel(kernel)
+        try:
+            g = run_batch(stride, S, T, tok, lay, mode, lam, windows=windows, V=V)
+        finally:
+            stride.stride_force_batch_kernel("auto")
+        assert g["status"] == 0
+        compare_rows(g, o)
+        compare_scan(g, o, lay, mode, lam)
