@@ -200,6 +200,35 @@ def test_steps_compact_per_rollout_lambda(stride):
 
 
 @pytest.mark.parametrize("form", ["masked", "compact"])
+@pytest.mark.parametrize("closes", ["every_token", "never"])
+def test_steps_turn_end_extremes(stride, form, closes):
+    """Every token closes its own turn (each step tests, turn means are
+    single log-probs), or no turn ever closes (turn mode never tests, so
+    nothing stops and every token is retained)."""
+    import torch
+
+    ring, B, steps, V = 3, 16, 120, 4099
+    S, T, tok, Sp, Tp = _ring(79, ring, B, V, V)
+    o_rows = oracle.row_logprobs(S, T, tok)
+    turn_end = np.full((steps, B), 1 if closes == "every_token" else 0, np.uint8)
+    # even rollouts: half their final never-stopping sum (they stop midway
+    # when tests happen); odd rollouts: out of reach
+    pre = oracle.new_rollouts(B)
+    for s in range(steps):
+        j = s % ring
+        oracle.step_update(pre, o_rows["logp_s"][j * B:(j + 1) * B], o_rows["logp_t"][j * B:(j + 1) * B],
+                           np.ones(B, np.uint8), 0, np.full(B, -np.inf))
+    lam = np.where(np.arange(B) % 2 == 0, 0.5 * oracle.rollouts_view(pre)["cum"], -1e6).astype(np.float32)
+    St, Tt = to_dev(Sp), to_dev(Tp)
+    tk = torch.from_numpy(tok).cuda()
+    r = run_steps(stride, St, Tt, tk, turn_end, ring, B, 0, lam, V, o_rows, form=form)
+    if closes == "never":
+        assert r["stopped"] == 0 and r["rows"] == steps * B
+    else:
+        assert r["stopped"] == B // 2
+
+
+@pytest.mark.parametrize("form", ["masked", "compact"])
 def test_steps_nan_thresholds_never_fire(stride, form):
     """A NaN entry of the per-rollout lambda never fires (the test is
     strict): that rollout never stops and every token it scores is
