@@ -92,6 +92,26 @@ def test_shards_combine_to_full_rows(stride, bounds_kind):
     assert np.max(np.abs(lt.cpu().numpy() - o["logp_t"])) <= LOGP_ATOL
 
 
+@pytest.mark.parametrize("V,n_shards", [(37, 37), (4099, 64)])
+def test_many_and_single_column_shards(stride, V, n_shards):
+    """Many shards: one column each (every shard but one misses the token),
+    or 64 shards of random widths (most of them starting off the 16-byte
+    grid); their partials merge to the oracle's log-probs."""
+    import torch
+
+    lay, S, T, tok = _case(64, V)
+    rng = np.random.default_rng(65)
+    cuts = np.sort(rng.choice(np.arange(1, V), size=n_shards - 1, replace=False)) if n_shards < V else np.arange(1, V)
+    bounds = [0] + [int(c) for c in cuts] + [V]
+    St, Tt = to_dev(S), to_dev(T)
+    tk = torch.from_numpy(tok).cuda()
+    ls, lt, status = _sharded_logprobs(stride, St, Tt, tk, bounds)
+    assert status == 0
+    o = oracle_batch(S, T, tok, lay, oracle.TURN_MEAN, -1e30)
+    assert np.max(np.abs(ls.cpu().numpy() - o["logp_s"])) <= LOGP_ATOL
+    assert np.max(np.abs(lt.cpu().numpy() - o["logp_t"])) <= LOGP_ATOL
+
+
 @pytest.mark.parametrize("mode", [0, 1])
 def test_scan_on_sharded_logprobs(stride, mode):
     import torch
