@@ -119,3 +119,59 @@ def test_multi_teacher_bad_rows_report(stride, case):
             workspace=torch.empty(stride.stride_score_batch_workspace_size(lay.rows), dtype=torch.uint8,
                                   device="cuda"))
     assert e.value.code == 3  # the row table needs 8 more bytes per row
+
+
+@pytest.mark.parametrize("kernel", ["auto", "stream", "split", "rows"])
+def test_eight_domains_scattered_rows(stride, kernel):
+    """The largest domain table (8 buffers of different lengths, two of them
+    unused), trajectories reading their teacher rows from random offsets of
+    their domain's buffer (ranges may overlap: the buffers are read only),
+    in one window and in three; against the oracle on the teacher rows
+    gathered by hand.  A ninth domain is rejected before any launch."""
+    import torch
+
+    rng = np.random.default_rng(88)
+    lens = [[int(rng.integers(2, 90)) for _ in range(int(rng.integers(1, 5)))] for _ in range(12)]
+    lay = synth.layout_from_turn_lengths(lens)
+    R, V = lay.rows, 2048
+    n_rows = np.diff(lay.traj_row_off)
+    S = synth.bf16_bits_from_f32(rng.standard_normal((R, V), dtype=np.float32) * np.float32(3.0))
+    dom = rng.choice([0, 1, 2, 4, 5, 7], size=lay.n_traj).astype(np.uint8)  # domains 3 and 6 unused
+    L = [int(n_rows.max()) + int(rng.integers(0, 400)) for _ in range(8)]
+    bufs = [synth.bf16_bits_from_f32(rng.standard_normal((L[d], V), dtype=np.float32) * np.float32(3.0))
+            for d in range(8)]
+    row0 = np.array([int(rng.integers(0, L[dom[i]] - n_rows[i] + 1)) for i in range(lay.n_traj)], np.int64)
+    T = np.concatenate([bufs[dom[i]][row0[i]:row0[i] + n_rows[i]] for i in range(lay.n_traj)])
+    tok = rng.integers(0, V, R).astype(np.int32)
+    o0 = oracle_batch_multi(S, T, tok, lay, -1e30)
+    lam = np.float32(np.median(o0["traj_cum"]))
+    o = oracle_batch_multi(S, T, tok, lay, lam)
+
+    def dev_bf16(a):
+        return torch.from_numpy(a.view(np.int16)).cuda().view(torch.bfloat16)
+
+    c = dict(lay=lay, S=dev_bf16(S), tok=torch.from_numpy(tok).cuda(), dom=dom, row0=row0,
+             T_dom=[dev_bf16(b) for b in bufs], lam=lam)
+    stride.stride_force_batch_kernel(kernel)
+    try:
+        for windows in ([(0, R)], [(0, R // 3), (R // 3, (2 * R) // 3), ((2 * R) // 3, R)]):
+            g = _run_multi(stride, c, windows)
+            assert g["status"] == 0
+            compare_rows(g, o)
+            compare_scan(g, o, lay, oracle.TURN_MEAN, lam)
+    finally:
+        stride.stride_force_batch_kernel("auto")
+    offs = [torch.from_numpy(a).cuda() for a in (lay.traj_row_off, lay.turn_row_off, lay.traj_turn_off)]
+    ws = torch.empty(stride.multi_teacher_workspace_size(R), dtype=torch.uint8, device="cuda")
+    with pytest.raises(stride.StrideError) as e:
+        stride.stride_score_batch_multi_teacher(c["S"], c["T_dom"] + [c["T_dom"][0]], torch.from_numpy(dom).cuda(),
+                                                torch.from_numpy(row0).cuda(), c["tok"], *offs, 0, R,
+                                                stride.TURN_MEAN, float(lam), stride.new_state(lay.n_traj),
+                                                workspace=ws)
+    assert e.value.code == stride.ERR_INVALID_ARG
+
+
+def oracle_batch_multi(S, T, tok, lay, lam):
+    from gpu_helpers import oracle_batch
+
+    return oracle_batch(S, T, tok, lay, oracle.TURN_MEAN, np.float32(lam))
