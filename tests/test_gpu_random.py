@@ -382,3 +382,41 @@ def test_tiny_windows(stride, kernel, width):
         assert g["status"] == 0
         compare_rows(g, o)
         compare_scan(g, o, lay, mode, lam)
+
+
+@pytest.mark.parametrize("kernel", ["auto", "stream", "split", "rows"])
+@pytest.mark.parametrize("f32", [False, True])
+def test_non_finite_logits(stride, kernel, f32):
+    """A NaN logit, a +inf logit (off the token, and at the token), and a row
+    of -inf logits: the row's log-probs are NaN (LSE NaN, or -inf with a -inf
+    gathered logit) exactly where the oracle's are, on both sides of the
+    pair; the other rows are untouched.  Kernels never trap on them."""
+    rng = np.random.default_rng(606 + f32)
+    lay = synth.layout_from_turn_lengths([[6, 5], [7], [4, 4, 4]])
+    R, V = lay.rows, 1000
+    S32 = rng.standard_normal((R, V), dtype=np.float32) * np.float32(2.0)
+    T32 = S32 + rng.standard_normal((R, V), dtype=np.float32)
+    tok = rng.integers(0, V, R).astype(np.int32)
+    S32[1, 5 if tok[1] != 5 else 6] = np.nan       # NaN in S, off the token
+    T32[3, 7 if tok[3] != 7 else 8] = np.inf       # +inf in T, off the token
+    T32[9, tok[9]] = np.inf                        # +inf at the token
+    S32[12, :] = -np.inf                           # a fully masked row
+    S32[20, 0] = np.nan
+    T32[20, 1] = np.inf                            # both sides
+    if f32:
+        S, T = S32, T32
+    else:
+        S, T = synth.bf16_bits_from_f32(S32), synth.bf16_bits_from_f32(T32)
+    o = oracle_batch(S, T, tok, lay, 1, np.float32(-1e30))
+    bad = [1, 3, 9, 12, 20]
+    for r in bad:
+        assert not (np.isfinite(o["logp_s"][r]) and np.isfinite(o["logp_t"][r])), r
+    good = np.setdiff1d(np.arange(R), bad)
+    assert np.isfinite(o["logp_s"][good]).all() and np.isfinite(o["logp_t"][good]).all()
+    stride.stride_force_batch_kernel(kernel)
+    try:
+        g = run_batch(stride, S, T, tok, lay, 1, np.float32(-1e30), V=V)
+    finally:
+        stride.stride_force_batch_kernel("auto")
+    assert g["status"] == 0
+    compare_rows(g, o)
