@@ -408,3 +408,42 @@ def test_compact_equals_masked_bitwise(stride, threads, C):
         stride.stride_force_step_shape(0, 0)
     assert np.array_equal(stride.state_to_numpy(st_m).view(np.uint8), stride.state_to_numpy(st_c).view(np.uint8))
     assert n_stops > 0
+
+
+@pytest.mark.parametrize("form", ["masked", "compact"])
+def test_step_non_finite_logits(stride, form):
+    """One step over rows with a NaN logit, a +inf logit (off and at the
+    token) and a row of -inf: log-probs NaN exactly where the oracle's are,
+    the clean rows untouched, no trap."""
+    import torch
+
+    rng = np.random.default_rng(91)
+    B, V = 6, 999
+    S32 = rng.standard_normal((B, V), dtype=np.float32) * np.float32(2.0)
+    T32 = S32 + rng.standard_normal((B, V), dtype=np.float32)
+    tok = rng.integers(0, V, B).astype(np.int32)
+    S32[0, 3 if tok[0] != 3 else 4] = np.nan
+    T32[1, 9 if tok[1] != 9 else 10] = np.inf
+    T32[2, tok[2]] = np.inf
+    S32[3, :] = -np.inf
+    S, T = synth.bf16_bits_from_f32(S32), synth.bf16_bits_from_f32(T32)
+    o = oracle.row_logprobs(S, T, tok)
+    St, Tt = to_dev(S), to_dev(T)
+    tk = torch.from_numpy(tok).cuda()
+    st = stride.new_state(B)
+    out = {k: torch.full((B,), 7.0, dtype=torch.float32, device="cuda") for k in ("logp_s", "logp_t", "opd")}
+    status = torch.zeros(1, dtype=torch.int32, device="cuda")
+    te = torch.zeros(B, dtype=torch.uint8, device="cuda")
+    if form == "masked":
+        stride.stride_score_step(St, Tt, tk, te, 1, -1e30, st, out=out, dev_status=status)
+    else:
+        idx = torch.arange(B, dtype=torch.int32, device="cuda")
+        stride.stride_score_step_compact(St, Tt, tk, te, idx, 1, -1e30, st, out=out, dev_status=status)
+    torch.cuda.synchronize()
+    assert int(status.item()) == 0
+    for k, ok in (("logp_s", "logp_s"), ("logp_t", "logp_t"), ("opd", "d")):
+        a, b = out[k].cpu().numpy().astype(np.float64), o[ok]
+        fin = np.isfinite(b)
+        assert np.array_equal(np.isfinite(a), fin), (k, a, b)
+        assert np.all(np.abs(a[fin] - b[fin]) <= LOGP_ATOL), k
+    assert np.isfinite(o["logp_t"][4:]).all() and np.isfinite(o["logp_s"][4:]).all()
