@@ -249,8 +249,9 @@ def check_opd_loss_golden(orc):
         rows = np.array([r for t in c["turns"] for r in t], np.float64)
         ls, lt = rows[:, 0], rows[:, 1]
         mode = oracle.TURN_MEAN if c["mode"] == "turn_mean" else oracle.TOKEN_SUM
+        cin = None if "cum_in" not in c else np.array([c["cum_in"]])
         o = orc.scan_batch(lt, ls - lt, lay.traj_row_off, lay.turn_row_off, lay.traj_turn_off, mode, c["lambda"],
-                           logp_s=ls)
+                           cum_in=cin, logp_s=ls)
         assert list(o["turn_sum_l"]) == c["turn_sum_l"], (c["name"], o["turn_sum_l"])
         assert o["traj_loss"][0] == c["loss"], (c["name"], o["traj_loss"])
         assert int(o["traj_loss_tokens"][0]) == c["loss_tokens"], c["name"]

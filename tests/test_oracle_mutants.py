@@ -41,6 +41,10 @@ MUTANTS = [
     ("loss_sign", "double term = logp_s ? logp_s[r - base] * dd : 0.0;", "double term = logp_s ? -logp_s[r - base] * dd : 0.0;"),
     ("loss_uses_teacher", "double term = logp_s ? logp_s[r - base] * dd : 0.0;", "double term = logp_s ? lt * dd : 0.0;"),
     ("loss_all_turns_retained", "int turn_retained = (st_turn < 0);", "int turn_retained = 1;"),
+    ("loss_first_turn_tested_against_start", "int turn_retained = (st_turn < 0);",
+     "int turn_retained = (st_turn < 0) && cum >= lambda[i];"),
+    ("loss_first_token_tested_against_start", "if (st_row < 0) {\n            loss += term;",
+     "if (st_row < 0 && cum >= lambda[i]) {\n            loss += term;"),
     ("loss_drops_trigger_token", "if (st_row < 0) {\n            loss += term;",
      "if (st_row < 0 && cum + lt >= lambda[i]) {\n            loss += term;"),
     ("profile_wrong_decile", "int64_t j = (10 * (r - a)) / n;", "int64_t j = (10 * (r - a)) / (n + 1);"),
