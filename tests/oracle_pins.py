@@ -231,7 +231,7 @@ def check_stop_rule_golden(orc):
         mode = oracle.TURN_MEAN if c["mode"] == "turn_mean" else oracle.TOKEN_SUM
         cin = None if "cum_in" not in c else np.array([c["cum_in"]])
         o = orc.scan_batch(lp, np.zeros_like(lp), lay.traj_row_off, lay.turn_row_off, lay.traj_turn_off,
-                           mode, c["lambda"], cum_in=cin)
+                           mode, float(c["lambda"]), cum_in=cin)  # "nan" / "inf" stored as strings
         assert list(o["turn_mean"]) == c["turn_mean"], (c["name"], o["turn_mean"])
         assert list(o["turn_cum"]) == c["turn_cum"], (c["name"], o["turn_cum"])
         assert int(o["stop_turn"][0]) == c["stop_turn"], (c["name"], o["stop_turn"])
@@ -250,8 +250,8 @@ def check_opd_loss_golden(orc):
         ls, lt = rows[:, 0], rows[:, 1]
         mode = oracle.TURN_MEAN if c["mode"] == "turn_mean" else oracle.TOKEN_SUM
         cin = None if "cum_in" not in c else np.array([c["cum_in"]])
-        o = orc.scan_batch(lt, ls - lt, lay.traj_row_off, lay.turn_row_off, lay.traj_turn_off, mode, c["lambda"],
-                           cum_in=cin, logp_s=ls)
+        o = orc.scan_batch(lt, ls - lt, lay.traj_row_off, lay.turn_row_off, lay.traj_turn_off, mode,
+                           float(c["lambda"]), cum_in=cin, logp_s=ls)
         assert list(o["turn_sum_l"]) == c["turn_sum_l"], (c["name"], o["turn_sum_l"])
         assert o["traj_loss"][0] == c["loss"], (c["name"], o["traj_loss"])
         assert int(o["traj_loss_tokens"][0]) == c["loss_tokens"], c["name"]
@@ -460,7 +460,7 @@ def check_step_golden(orc):
         lay = layout_from_turn_lengths([[len(t) for t in turns]])
         lp = np.array([v for t in turns for v in t], np.float64)
         mode = oracle.TURN_MEAN if c["mode"] == "turn_mean" else oracle.TOKEN_SUM
-        st, _, _ = _run_steps(orc, lay, lp, np.zeros_like(lp), mode, c["lambda"])
+        st, _, _ = _run_steps(orc, lay, lp, np.zeros_like(lp), mode, float(c["lambda"]))
         assert st[0].stop_turn == c["stop_turn"] and st[0].stop_row == c["stop_row"], c["name"]
 
 
