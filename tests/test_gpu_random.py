@@ -420,3 +420,71 @@ def test_non_finite_logits(stride, kernel, f32):
         stride.stride_force_batch_kernel("auto")
     assert g["status"] == 0
     compare_rows(g, o)
+
+
+def _mixed_case(seed):
+    """A layout mixing the degenerate cases: empty trajectories, one-row
+    turns and long turns; per-trajectory lambda finite, +inf, -inf or NaN;
+    starting sums 0 or carried (some below lambda); random window cuts;
+    both dtypes, padded or exact strides."""
+    rng = np.random.default_rng(20_000 + seed)
+    lens = []
+    for _ in range(int(rng.integers(3, 12))):
+        u = rng.random()
+        if u < 0.15:
+            lens.append([])
+        else:
+            lens.append([1 if rng.random() < 0.25 else int(rng.integers(2, 400 if u < 0.3 else 60))
+                         for _ in range(int(rng.integers(1, 6)))])
+    if all(len(t) == 0 for t in lens):
+        lens.append([int(rng.integers(1, 30))])
+    lay = synth.layout_from_turn_lengths(lens)
+    R = lay.rows
+    V = int(rng.choice([129, 1000, 4099]))
+    f32 = bool(rng.random() < 0.5)
+    ld = V + (int(rng.integers(1, 9)) if rng.random() < 0.4 else 0)
+    mode = int(rng.integers(0, 2))
+    S32 = rng.standard_normal((R, V), dtype=np.float32) * np.float32(rng.uniform(1.0, 4.0))
+    T32 = S32 + rng.standard_normal((R, V), dtype=np.float32) * np.float32(rng.uniform(0.2, 1.5))
+    if f32:
+        S, T, fill = S32, T32, np.float32(np.nan)
+    else:
+        S = synth.bf16_bits_from_f32(S32)
+        T = synth.bf16_bits_from_f32(synth.f32_from_bf16_bits(S) + (T32 - S32))
+        fill = 0x7FC0
+    tok = rng.integers(0, V, R).astype(np.int32)
+    cuts = sorted(set([0, R] + [int(x) for x in rng.integers(1, R, size=int(rng.integers(0, 5)))])) if R > 1 else [0, R]
+    return rng, lay, S, T, tok, V, ld, mode, list(zip(cuts[:-1], cuts[1:])), fill
+
+
+@pytest.mark.parametrize("kernel", ["auto", "stream", "split", "rows"])
+@pytest.mark.parametrize("seed", list(range(24)))
+def test_mixed_degenerate_layouts(stride, seed, kernel):
+    import torch
+
+    import oracle
+
+    rng, lay, S, T, tok, V, ld, mode, windows, fill = _mixed_case(seed)
+    o0 = oracle_batch(S, T, tok, lay, mode, np.float32(-1e30))
+    lam = _lambda(o0, lay, mode, rng)
+    special = rng.random(lay.n_traj)
+    lam[special < 0.1] = np.float32(np.inf)
+    lam[(special >= 0.1) & (special < 0.2)] = np.float32(-np.inf)
+    lam[(special >= 0.2) & (special < 0.3)] = np.float32(np.nan)
+    cum0 = np.where(rng.random(lay.n_traj) < 0.3, rng.uniform(-80.0, 0.0, lay.n_traj), 0.0)
+    o = oracle_batch(S, T, tok, lay, mode, lam)
+    o.update(oracle.scan_batch(o["logp_t"], o["d"], lay.traj_row_off, lay.turn_row_off, lay.traj_turn_off, mode,
+                               lam.astype(np.float64), cum_in=cum0, logp_s=o["logp_s"]))
+    st = stride.new_state(lay.n_traj)
+    h = stride.state_to_numpy(st)[: lay.n_traj].copy()
+    h["cum"] = cum0
+    st[: lay.n_traj].copy_(torch.from_numpy(h.view(np.uint8).reshape(lay.n_traj, -1)).cuda())
+    Sp, Tp = (S, T) if ld == V else (pad_cols(S, ld, fill), pad_cols(T, ld, fill))
+    stride.stride_force_batch_kernel(kernel)
+    try:
+        g = run_batch(stride, Sp, Tp, tok, lay, mode, lam, windows=windows, V=V, state=st)
+    finally:
+        stride.stride_force_batch_kernel("auto")
+    assert g["status"] == 0
+    compare_rows(g, o)
+    compare_scan(g, o, lay, mode, lam)
