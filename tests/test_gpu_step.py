@@ -42,14 +42,15 @@ def _ring(seed, ring, B, V, ld):
     return S, T, tok, Sp, Tp
 
 
-def run_steps(stride, St, Tt, tk, turn_end, ring, B, mode, lam, V, o_rows, form="masked"):
+def run_steps(stride, St, Tt, tk, turn_end, ring, B, mode, lam, V, o_rows, form="masked", cum0=None):
     """Run len(turn_end) steps; step s reads slab s % ring (rollout b's row is
     row b of the slab).  form = "masked": stride_score_step over all B rows;
     "compact": stride_score_step_compact over the rows of the rollouts that
     have not stopped, gathered from the slab as a rollout engine that
     batches only live sequences would hand them over (the live set is the
     GPU's own, from stopped_now).  lam: a scalar or a float32 array [B].
-    Returns a summary of the run."""
+    cum0: optional starting running sums [B] (a carried offset), set in the
+    GPU state and in the oracle's.  Returns a summary of the run."""
     import torch
 
     steps = turn_end.shape[0]
@@ -59,6 +60,12 @@ def run_steps(stride, St, Tt, tk, turn_end, ring, B, mode, lam, V, o_rows, form=
     st = stride.new_state(B)
     ost, shadow = oracle.new_rollouts(B), oracle.new_rollouts(B)
     ov, sv = oracle.rollouts_view(ost), oracle.rollouts_view(shadow)
+    if cum0 is not None:
+        h = stride.state_to_numpy(st)[:B].copy()
+        h["cum"] = cum0
+        st[:B].copy_(torch.from_numpy(h.view(np.uint8).reshape(B, -1)).cuda())
+        ov["cum"][:] = cum0
+        sv["cum"][:] = cum0
     out = {k: torch.empty(B, dtype=torch.float32, device="cuda") for k in ("logp_s", "logp_t", "opd")}
     sn = torch.empty(B, dtype=torch.uint8, device="cuda")
     tout = torch.empty((B, stride.TURN_STATS_DTYPE.itemsize), dtype=torch.uint8, device="cuda")
@@ -226,6 +233,33 @@ def test_steps_turn_end_extremes(stride, form, closes):
         assert r["stopped"] == 0 and r["rows"] == steps * B
     else:
         assert r["stopped"] == B // 2
+
+
+@pytest.mark.parametrize("form", ["masked", "compact"])
+@pytest.mark.parametrize("seed", list(range(6)))
+def test_steps_mixed_degenerate(stride, form, seed):
+    """Seeded decode runs mixing per-rollout lambda finite, +inf, -inf and
+    NaN, carried starting sums (some already below lambda: those stop at
+    their first test), random turn ends, both modes."""
+    import torch
+
+    rng = np.random.default_rng(300 + seed)
+    ring, B, steps = 3, int(rng.integers(5, 40)), int(rng.integers(40, 160))
+    V = int(rng.choice([257, 4099]))
+    mode = int(rng.integers(0, 2))
+    S, T, tok, Sp, Tp = _ring(400 + seed, ring, B, V, V)
+    o_rows = oracle.row_logprobs(S, T, tok)
+    turn_end = (rng.random((steps, B)) < rng.uniform(0.02, 0.3)).astype(np.uint8)
+    scale = -4.0 * steps if mode == oracle.TOKEN_SUM else -4.0 * max(1.0, turn_end.sum(0).mean())
+    lam = (scale * rng.uniform(0.2, 1.0, B)).astype(np.float32)
+    u = rng.random(B)
+    lam[u < 0.15] = np.float32(np.inf)
+    lam[(u >= 0.15) & (u < 0.3)] = np.float32(-np.inf)
+    lam[(u >= 0.3) & (u < 0.45)] = np.float32(np.nan)
+    cum0 = np.where(rng.random(B) < 0.3, rng.uniform(1.5, 3.0, B) * np.where(np.isfinite(lam), lam, -10.0), 0.0)
+    St, Tt = to_dev(Sp), to_dev(Tp)
+    tk = torch.from_numpy(tok).cuda()
+    run_steps(stride, St, Tt, tk, turn_end, ring, B, mode, lam, V, o_rows, form=form, cum0=cum0)
 
 
 @pytest.mark.parametrize("form", ["masked", "compact"])
