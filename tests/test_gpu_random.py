@@ -488,3 +488,50 @@ def test_mixed_degenerate_layouts(stride, seed, kernel):
     assert g["status"] == 0
     compare_rows(g, o)
     compare_scan(g, o, lay, mode, lam)
+
+
+@pytest.mark.parametrize("seed", list(range(24)))
+def test_mixed_degenerate_scan_on_logprobs(stride, seed):
+    """The mixed layouts through stride_scan_logprobs (the tiled scan on its
+    own: 256-row tiles by ticket, one lookback per tile), fed the oracle's
+    log-probs rounded to fp32, with the same thresholds and starting sums."""
+    import torch
+
+    import oracle
+
+    rng, lay, S, T, tok, V, ld, mode, windows, fill = _mixed_case(seed)
+    o_rows = oracle_batch(S, T, tok, lay, mode, np.float32(-1e30))
+    lps = o_rows["logp_s"].astype(np.float32)
+    lpt = o_rows["logp_t"].astype(np.float32)
+    d = lps.astype(np.float64) - lpt.astype(np.float64)
+    o0 = oracle.scan_batch(lpt.astype(np.float64), d, lay.traj_row_off, lay.turn_row_off, lay.traj_turn_off, mode,
+                           np.float64(-1e30), logp_s=lps.astype(np.float64))
+    lam = _lambda(o0, lay, mode, rng)
+    special = rng.random(lay.n_traj)
+    lam[special < 0.1] = np.float32(np.inf)
+    lam[(special >= 0.1) & (special < 0.2)] = np.float32(-np.inf)
+    lam[(special >= 0.2) & (special < 0.3)] = np.float32(np.nan)
+    cum0 = np.where(rng.random(lay.n_traj) < 0.3, rng.uniform(-80.0, 0.0, lay.n_traj), 0.0)
+    o = oracle.scan_batch(lpt.astype(np.float64), d, lay.traj_row_off, lay.turn_row_off, lay.traj_turn_off, mode,
+                          lam.astype(np.float64), cum_in=cum0, logp_s=lps.astype(np.float64))
+    o.update(logp_t=lpt.astype(np.float64), logp_s=lps.astype(np.float64), d=d)
+    dev = "cuda"
+    R = lay.rows
+    offs = [torch.from_numpy(a).to(dev) for a in (lay.traj_row_off, lay.turn_row_off, lay.traj_turn_off)]
+    st = stride.new_state(lay.n_traj)
+    h = stride.state_to_numpy(st)[: lay.n_traj].copy()
+    h["cum"] = cum0
+    st[: lay.n_traj].copy_(torch.from_numpy(h.view(np.uint8).reshape(lay.n_traj, -1)).cuda())
+    ts = stride.new_turn_stats(lay.n_turns)
+    prof = stride.new_profile(dev)
+    status = torch.zeros(1, dtype=torch.int32, device=dev)
+    ws = torch.empty(stride.stride_score_batch_workspace_size(max(1, R)), dtype=torch.uint8, device=dev)
+    lps_d, lpt_d, lam_d = (torch.from_numpy(a).to(dev) for a in (lps, lpt, lam))
+    for a, b in windows:
+        stride.stride_scan_logprobs(lps_d[a:b], lpt_d[a:b], *offs, a, b, mode, lam_d, st, turn_stats=ts,
+                                    dev_status=status, workspace=ws, profile=prof)
+    torch.cuda.synchronize()
+    assert int(status.item()) == 0
+    g = {"state": stride.state_to_numpy(st)[: lay.n_traj], "turn_stats": stride.turn_stats_to_numpy(ts)[: lay.n_turns],
+         "profile": prof.cpu().numpy()}
+    compare_scan(g, o, lay, mode, lam)
