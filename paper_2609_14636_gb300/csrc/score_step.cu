@@ -305,6 +305,7 @@ Shape choose_shape(int64_t rows, int sms) {
   const int ft = g_force_threads.load(std::memory_order_relaxed);
   const int fc = g_force_cluster.load(std::memory_order_relaxed);
   if (ft > 0 || fc > 0) return Shape{ft > 0 ? ft : kStepThreadsSmall, fc > 0 ? fc : 1};
+  if (rows <= 4) return Shape{kStepThreadsLarge, 16};
   if (rows <= 32) return Shape{kStepThreadsLarge, 8};
   const int64_t fill = (int64_t)sms * 8 * 85 / 100;  // 128-thread CTAs in 0.85 of a wave
   int64_t c = fill / rows;
