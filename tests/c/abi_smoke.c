@@ -1,4 +1,5 @@
 /* A C99 caller of libstride.so: only include/stride.h and the CUDA runtime.
+ * (Also three decode steps on the same rows, and the vocabulary limit.)
  *
  * Scores 9 rows of uniform fp32 logits (student = teacher = 0 over V = 1000)
  * in two trajectories (turns of 3 + 2 rows, and 4 rows) under the token-sum
@@ -133,6 +134,36 @@ int main(void) {
   CHECK_CUDA(cudaMemcpy(&ks, dks, sizeof ks, cudaMemcpyDeviceToHost));
   CHECK_CUDA(cudaMemcpy(&km, dkm, sizeof km, cudaMemcpyDeviceToHost));
   EXPECT(ks == 1 && km == 2);
+
+  /* three decode steps over rows 0-1 as two rollouts (token-sum rule,
+   * lambda = -20): each step adds -ln V, so the third (-20.72) stops both,
+   * and every scored token is retained */
+  enum { B = 2 };
+  stride_scan_state* dst2;
+  unsigned char *dte, *dsn;
+  CHECK_CUDA(cudaMalloc((void**)&dst2, sizeof(stride_scan_state) * B));
+  CHECK_CUDA(cudaMalloc((void**)&dte, B));
+  CHECK_CUDA(cudaMalloc((void**)&dsn, B));
+  CHECK_CUDA(cudaMemset(dte, 0, B));
+  EXPECT(stride_state_init(dst2, B, NULL) == STRIDE_OK);
+  unsigned char sn[B];
+  for (int s = 0; s < 3; ++s) {
+    EXPECT(stride_score_step(dS, dT, STRIDE_DTYPE_F32, V, V, dtok, dte, B, STRIDE_STOP_TOKEN_SUM, NULL, -20.f,
+                             dst2, &out, dsn, NULL, dstatus, NULL) == STRIDE_OK);
+    CHECK_CUDA(cudaMemcpy(sn, dsn, sizeof sn, cudaMemcpyDeviceToHost));
+    for (int b = 0; b < B; ++b) EXPECT(sn[b] == (s == 2));
+  }
+  stride_scan_state st2[B];
+  CHECK_CUDA(cudaMemcpy(st2, dst2, sizeof st2, cudaMemcpyDeviceToHost));
+  for (int b = 0; b < B; ++b) {
+    EXPECT(st2[b].stopped && st2[b].stop_row == 2 && st2[b].rows_seen == 3 && st2[b].loss_tokens == 3);
+    EXPECT(fabs(st2[b].cum + 3.0 * lnv) <= 1e-5 * 3.0 * lnv);
+  }
+
+  /* the vocabulary limit is checked on the host: one column more is refused */
+  EXPECT(stride_score_batch(dS, dT, STRIDE_DTYPE_F32, (int64_t)STRIDE_MAX_VOCAB + 1, (int64_t)STRIDE_MAX_VOCAB + 1,
+                            dtok, dtraj, dturn, dturn_off32, NTRAJ, NTURN, 0, R, STRIDE_STOP_TOKEN_SUM, NULL, -20.f,
+                            dstate, &out, dts, NULL, dstatus, dws, ws_bytes, NULL) == STRIDE_ERR_INVALID_ARG);
   printf("abi_smoke ok\n");
   return 0;
 }

@@ -1,7 +1,8 @@
 """A C program (tests/c/abi_smoke.c) calls libstride.so through
 include/stride.h alone: it builds and links on the CPU, and on a GPU it
 scores uniform-logit rows, checks the closed-form log-probs, the stop rule
-and the loss, and makes one restart choice."""
+and the loss, makes one restart choice, runs three decode steps, and sees
+one column past the vocabulary limit refused."""
 import shutil
 import subprocess
 from pathlib import Path
