@@ -182,8 +182,9 @@ struct TileElem {
   int flags;
 };
 
-// A prefix over tiles (the lookback's result, a row's inclusive and
-// exclusive values): fp64 throughout.
+// A prefix over tiles as the lookback folds it: fp64 throughout.  (A row's
+// inclusive and exclusive values, and the cluster form's fold, use TileElem:
+// the stop sum fp64, the open-turn sums fp32.)
 struct PreElem {
   double c, st, sd, sl;
 };
