@@ -172,10 +172,12 @@ constexpr int kRestartSum = 2;   // c restarts (a seeded row)
 // A row's element inside a tile.  The running stop sum c is fp64 (the stop
 // rule compares it with lambda); the open-turn sums of log pi_T, d and the
 // loss term are fp32 inside the tile (at most kScanTileRows terms each,
-// summed in a tree: relative error a few 1e-7 of the summed magnitudes) and
-// fp64 again once combined with the tile's prefix.  GB300 runs FP64 at 1/64
-// of the FP32 rate, and the tile scans' fp64 adds were what a small window's
-// scan waited on (a 512-row window in one CTA: 6.6 us for the block scan).
+// summed in a tree: relative error a few 1e-7 of the summed magnitudes), in
+// the cluster form's fold of at most 16 tile aggregates, and where the
+// tile's prefix meets a row; the lookback's prefix over tiles and every
+// stored sum are fp64.  GB300 runs FP64 at 1/64 of the FP32 rate, and the
+// tile scans' fp64 adds were what a small window's scan waited on (a
+// 512-row window in one CTA: 6.6 us for the block scan).
 struct TileElem {
   double c;
   float st, sd, sl;
